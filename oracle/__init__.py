@@ -1,0 +1,192 @@
+"""fp64 CPU oracle of ESPACE's projected linear layer -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the benchmark's ``cpu_baseline`` /
+``--impl reference`` legs may import this package. The product library never does, and the
+oracle never imports the product: the two share no code. The arithmetic lives in the plain
+C file ``espace_oracle.c`` (built by ``oracle.build``); this module only marshals numpy
+arrays and chains the steps in the order the paper states them:
+
+* ``autocorr_sum``      Eq. 4, the sum of x x^T over calibration tokens (no centering);
+* ``eigh``              the EVD of Sec. 3.1 by cyclic Jacobi, eigenvalues decreasing;
+* ``build_projection``  Thm. 1: P = the L principal eigenvectors of C = S / n, then bf16;
+* ``fold``              W' = P^T W (Sec. 2.2), bf16;
+* ``project``           Z = P^T X, rounded to bf16 (the rank-L intermediate of Eq. 3);
+* ``contract``          Y = W'^T Z (Eq. 3), fp64;
+* ``forward``           project then contract: the projected linear layer of Eq. 3;
+* ``dense``             Y = W^T X (Eq. 1);
+* ``reconstruct`` / ``projection_mse``  Eq. 5 and Eq. 6;
+* ``autocorr_normalized_sum``           Cor. 1's input-normalized autocorrelation.
+
+Layout: tokens are rows (``X`` is ``[N, K]``), ``W`` is ``[M, K]`` as in ``nn.Linear``,
+``P`` is ``[K, L]``, ``W'`` is ``[L, M]``, ``Z`` is ``[N, L]`` and ``Y`` is ``[N, M]``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from .build import build, library_path
+
+_lib = None
+_dp = ctypes.POINTER(ctypes.c_double)
+_i64 = ctypes.c_int64
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        path = library_path()
+        if not os.path.exists(path):
+            build()
+        lib = ctypes.CDLL(path)
+        lib.oracle_bf16_round.restype = ctypes.c_double
+        lib.oracle_bf16_round.argtypes = [ctypes.c_double]
+        lib.oracle_bf16_round_array.argtypes = [_dp, _i64]
+        lib.oracle_autocorr_sum.argtypes = [_dp, _i64, _i64, _dp]
+        lib.oracle_autocorr_normalized_sum.argtypes = [_dp, _i64, _i64, _dp]
+        lib.oracle_jacobi_eigh.restype = ctypes.c_int
+        lib.oracle_jacobi_eigh.argtypes = [_dp, _i64, _dp, _dp, ctypes.c_int, ctypes.c_double]
+        lib.oracle_fold.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp, ctypes.c_int]
+        lib.oracle_project.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp, ctypes.c_int]
+        lib.oracle_contract.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp]
+        lib.oracle_dense.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp]
+        lib.oracle_reconstruct.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp]
+        lib.oracle_projection_mse.restype = ctypes.c_double
+        lib.oracle_projection_mse.argtypes = [_dp, _dp, _i64, _i64, _i64]
+        _lib = lib
+    return _lib
+
+
+def _f64(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float64))
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(_dp)
+
+
+def bf16_round(a) -> np.ndarray:
+    """Round every entry to the nearest bf16 value (ties to even), returned as fp64."""
+    out = _f64(a).copy()
+    _load().oracle_bf16_round_array(_ptr(out), out.size)
+    return out
+
+
+def autocorr_sum(X, S: np.ndarray | None = None) -> np.ndarray:
+    """Eq. 4: ``S + sum_t x_t x_t^T`` over the token rows of ``X`` ([n, K])."""
+    X = _f64(X)
+    n, K = X.shape
+    S = np.zeros((K, K)) if S is None else _f64(S).copy()
+    _load().oracle_autocorr_sum(_ptr(X), n, K, _ptr(S))
+    return S
+
+
+def autocorr_normalized_sum(X, S: np.ndarray | None = None) -> np.ndarray:
+    """Cor. 1: ``S + sum_t (x_t/|x_t|)(x_t/|x_t|)^T``."""
+    X = _f64(X)
+    n, K = X.shape
+    S = np.zeros((K, K)) if S is None else _f64(S).copy()
+    _load().oracle_autocorr_normalized_sum(_ptr(X), n, K, _ptr(S))
+    return S
+
+
+def eigh(C, max_sweeps: int = 60, tol: float = 1e-15):
+    """Symmetric EVD by cyclic Jacobi: ``(w, V, sweeps)`` with ``w`` decreasing and
+    ``C = V diag(w) V^T``."""
+    A = _f64(C).copy()
+    K = A.shape[0]
+    w = np.zeros(K)
+    V = np.zeros((K, K))
+    sweeps = _load().oracle_jacobi_eigh(_ptr(A), K, _ptr(w), _ptr(V), max_sweeps, tol)
+    return w, V, sweeps
+
+
+def normalize_signs(P: np.ndarray) -> np.ndarray:
+    """Flip each column so that its entry of largest magnitude (lowest index on ties) is
+    positive. Eigenvectors are defined up to sign; Y does not depend on the choice."""
+    P = _f64(P).copy()
+    for j in range(P.shape[1]):
+        i = int(np.argmax(np.abs(P[:, j])))
+        if P[i, j] < 0:
+            P[:, j] = -P[:, j]
+    return P
+
+
+def build_projection(S, n: int, L: int):
+    """Thm. 1: ``C = S / n``; ``P`` = its ``L`` principal eigenvectors (fp64, signs
+    normalized) and ``P_b`` = ``P`` rounded to bf16. Returns ``(P, P_b, w, sweeps)``."""
+    C = _f64(S) / float(n)
+    w, V, sweeps = eigh(C)
+    P = normalize_signs(V[:, :L])
+    return P, bf16_round(P), w, sweeps
+
+
+def fold(P, W, round_bf16: bool = True) -> np.ndarray:
+    """``W' = P^T W`` as ``[L, M]`` from ``P`` ([K, L]) and ``W`` ([M, K])."""
+    P, W = _f64(P), _f64(W)
+    K, L = P.shape
+    M = W.shape[0]
+    assert W.shape[1] == K
+    Wf = np.zeros((L, M))
+    _load().oracle_fold(_ptr(P), _ptr(W), K, M, L, _ptr(Wf), int(round_bf16))
+    return Wf
+
+
+def project(X, P, round_bf16: bool = True) -> np.ndarray:
+    """``Z = P^T X`` stored token-major as ``[N, L]``."""
+    X, P = _f64(X), _f64(P)
+    N, K = X.shape
+    L = P.shape[1]
+    assert P.shape[0] == K
+    Z = np.zeros((N, L))
+    _load().oracle_project(_ptr(X), _ptr(P), N, K, L, _ptr(Z), int(round_bf16))
+    return Z
+
+
+def contract(Z, Wf) -> np.ndarray:
+    """``Y = W'^T Z`` as ``[N, M]`` in fp64."""
+    Z, Wf = _f64(Z), _f64(Wf)
+    N, L = Z.shape
+    M = Wf.shape[1]
+    assert Wf.shape[0] == L
+    Y = np.zeros((N, M))
+    _load().oracle_contract(_ptr(Z), _ptr(Wf), N, L, M, _ptr(Y))
+    return Y
+
+
+def forward(X, P_b, W, Wf=None, round_bf16: bool = True):
+    """The projected linear layer of Eq. 3: ``(Y, Z, W')``."""
+    if Wf is None:
+        Wf = fold(P_b, W, round_bf16)
+    Z = project(X, P_b, round_bf16)
+    return contract(Z, Wf), Z, Wf
+
+
+def dense(X, W) -> np.ndarray:
+    """Eq. 1: ``Y = W^T X`` as ``[N, M]``."""
+    X, W = _f64(X), _f64(W)
+    N, K = X.shape
+    M = W.shape[0]
+    assert W.shape[1] == K
+    Y = np.zeros((N, M))
+    _load().oracle_dense(_ptr(X), _ptr(W), N, K, M, _ptr(Y))
+    return Y
+
+
+def reconstruct(X, P) -> np.ndarray:
+    """Eq. 5: ``x~ = sum_i <p_i, x> p_i`` for each token row."""
+    X, P = _f64(X), _f64(P)
+    N, K = X.shape
+    L = P.shape[1]
+    Xt = np.zeros((N, K))
+    _load().oracle_reconstruct(_ptr(X), _ptr(P), N, K, L, _ptr(Xt))
+    return Xt
+
+
+def projection_mse(X, P) -> float:
+    """Eq. 6: sample mean of ``||x - x~||^2``."""
+    X, P = _f64(X), _f64(P)
+    N, K = X.shape
+    return float(_load().oracle_projection_mse(_ptr(X), _ptr(P), N, K, P.shape[1]))

@@ -1,0 +1,270 @@
+"""Pins the fp64 oracle to facts the paper and plain mathematics fix (no GPU needed).
+
+The oracle is trusted only through these checks: closed forms, brute force on tiny inputs
+(pure-Python loops), identities the paper proves (Thm. 1's MSE formula, Eq. 3's
+associativity, Prop. 1's bounds, L = K being exact), and library routines (numpy's LAPACK
+eigh, torch's bf16 cast) used as independent witnesses.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+
+def rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- bf16 round-to-nearest-even
+
+def _all_bf16_values():
+    bits = torch.arange(0, 1 << 16, dtype=torch.int32).to(torch.int16)
+    vals = bits.view(torch.bfloat16).to(torch.float64).numpy()
+    pat = np.arange(1 << 16)
+    ok = np.isfinite(vals) & (vals >= 0) & (pat < 0x8000)
+    return vals[ok], pat[ok]
+
+
+def test_bf16_round_matches_torch_on_fp32_inputs():
+    r = rng(1)
+    u = r.integers(0, 1 << 32, size=1_000_000, dtype=np.uint64).astype(np.uint32)
+    x = u.view(np.float32)
+    x = x[np.isfinite(x)]
+    # exact ties: a bf16 value plus half of its spacing (representable in fp32)
+    base = (r.integers(0, 1 << 16, size=20000, dtype=np.uint32) << 16).view(np.float32)
+    base = base[np.isfinite(base) & (np.abs(base) < 1e38)]
+    tie = (base.view(np.uint32) | np.uint32(0x8000)).view(np.float32)
+    x = np.concatenate([x, tie, np.array([0.0, -0.0, 1e-40, -1e-40, 3.4e38, -3.4e38,
+                                          np.inf, -np.inf], dtype=np.float32)])
+    want = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    got = oracle.bf16_round(x.astype(np.float64))
+    assert np.array_equal(got, want)
+
+
+def test_bf16_round_matches_nearest_in_table_of_all_bf16_values():
+    vals, pat = _all_bf16_values()
+    order = np.argsort(vals, kind="stable")
+    vals, pat = vals[order], pat[order]
+    keep = np.concatenate([[True], np.diff(vals) > 0])     # +0 and -0 collapse
+    vals, pat = vals[keep], pat[keep]
+    r = rng(2)
+    x = np.concatenate([
+        np.exp(r.uniform(-300, 88, size=200000)),          # wide dynamic range, fp64 values
+        r.uniform(0, 1e-38, size=20000),                   # subnormal range of bf16
+        (vals[1:2000] + vals[:1999]) / 2.0,                # exact midpoints -> ties to even
+    ])
+    got = oracle.bf16_round(x)
+    idx = np.clip(np.searchsorted(vals, x), 1, len(vals) - 1)
+    lo, hi = vals[idx - 1], vals[idx]
+    dlo, dhi = x - lo, hi - x
+    pick_hi = (dhi < dlo) | ((dhi == dlo) & (pat[idx] % 2 == 0))
+    want = np.where(pick_hi, hi, lo)
+    assert np.array_equal(got, want)
+    assert np.array_equal(oracle.bf16_round(-x), -want)
+
+
+# ---------------------------------------------------------------- autocorrelation (Eq. 4)
+
+def test_autocorr_brute_force():
+    r = rng(3)
+    X = r.standard_normal((7, 5))
+    S = oracle.autocorr_sum(X)
+    for i in range(5):
+        for j in range(5):
+            acc = 0.0
+            for t in range(7):
+                acc += X[t][i] * X[t][j]
+            assert abs(S[i, j] - acc) <= 1e-14 * (1 + abs(acc))
+
+
+def test_autocorr_invariants():
+    r = rng(4)
+    X = r.standard_normal((300, 12)) * np.linspace(0.1, 3.0, 12)
+    S = oracle.autocorr_sum(X)
+    assert np.array_equal(S, S.T)
+    # trace(C) = mean ||x||^2
+    assert math.isclose(np.trace(S) / 300, np.mean(np.sum(X * X, axis=1)), rel_tol=1e-12)
+    # shard invariance: accumulating two shards equals accumulating the whole
+    S2 = oracle.autocorr_sum(X[170:], oracle.autocorr_sum(X[:170]))
+    assert np.allclose(S, S2, rtol=1e-13, atol=1e-12)
+    # positive semi-definite
+    w = np.linalg.eigvalsh(S)
+    assert w.min() >= -1e-12 * w.max()
+
+
+def test_normalized_autocorr_is_autocorr_of_unit_vectors():
+    r = rng(5)
+    X = r.standard_normal((50, 9)) * 7.0
+    X[3] = 0.0                                   # a zero token contributes nothing
+    U = X.copy()
+    nz = np.linalg.norm(U, axis=1) > 0
+    U[nz] /= np.linalg.norm(U[nz], axis=1, keepdims=True)
+    Shat = oracle.autocorr_normalized_sum(X)
+    assert np.allclose(Shat, oracle.autocorr_sum(U), rtol=1e-13, atol=1e-13)
+    assert math.isclose(np.trace(Shat), 49.0, rel_tol=1e-13)
+
+
+# ---------------------------------------------------------------- Jacobi EVD
+
+def test_eigh_2x2_closed_form():
+    a, b, c = 2.5, -1.25, 0.75
+    w, V, _ = oracle.eigh(np.array([[a, b], [b, c]]))
+    mid, rad = (a + c) / 2, math.hypot((a - c) / 2, b)
+    assert np.allclose(w, [mid + rad, mid - rad], rtol=0, atol=1e-15)
+    # first eigenvector solves (A - l1 I) v = 0
+    v = V[:, 0]
+    assert abs((a - w[0]) * v[0] + b * v[1]) < 1e-14
+
+
+def test_eigh_diagonal_and_sorting():
+    d = np.array([0.5, 3.0, -1.0, 2.0])
+    w, V, sweeps = oracle.eigh(np.diag(d))
+    assert sweeps == 0
+    assert np.array_equal(w, np.sort(d)[::-1])
+    assert np.array_equal(np.abs(V), np.abs(np.eye(4)[:, np.argsort(-d)]))
+
+
+@pytest.mark.parametrize("K", [17, 64, 150])
+def test_eigh_reconstruction_and_lapack(K):
+    r = rng(K)
+    B = r.standard_normal((K, K))
+    C = B @ B.T / K + np.diag(np.linspace(0, 1, K))
+    w, V, sweeps = oracle.eigh(C)
+    assert sweeps < 60
+    assert np.all(np.diff(w) <= 0)
+    assert np.allclose(V.T @ V, np.eye(K), atol=1e-12)
+    assert np.allclose(V @ np.diag(w) @ V.T, C, atol=1e-12 * np.abs(C).max())
+    ref = np.linalg.eigh(C)[0][::-1]
+    assert np.allclose(w, ref, rtol=0, atol=1e-12 * ref[0])
+    # well-separated spectrum: eigenvectors agree with LAPACK up to sign
+    wl, Vl = np.linalg.eigh(C)
+    Vl = Vl[:, ::-1]
+    gaps = np.minimum(np.abs(np.diff(ref, prepend=np.inf)), np.abs(np.diff(ref, append=-np.inf)))
+    sep = gaps > 1e-6 * ref[0]
+    dots = np.abs(np.sum(V * Vl, axis=0))
+    assert np.all(dots[sep] > 1 - 1e-9)
+
+
+def test_population_spectrum_power_law():
+    """With unit channel scales, no outliers and n >> K, the eigenvalues of C approach the
+    generator's s_i^2 = i^-1.6."""
+    K, n = 16, 200000
+    model = synth.ActivationModel(K, seed=11, outliers=0, lognormal_sigma=0.0)
+    X = model.sample_f32(n).astype(np.float64)
+    w, _, _ = oracle.eigh(oracle.autocorr_sum(X) / n)
+    target = np.arange(1, K + 1) ** -1.6
+    assert np.allclose(w, target, rtol=0.03)
+
+
+# ---------------------------------------------------------------- Thm. 1 and Eq. 5-6
+
+def _calib(K=24, n=4000, seed=6):
+    model = synth.ActivationModel(K, seed=seed, outliers=2, lognormal_sigma=0.5)
+    return model.sample_f32(n).astype(np.float64)
+
+
+def test_theorem1_mse_equals_discarded_eigenvalues():
+    X = _calib()
+    n, K = X.shape
+    for L in (1, 5, 12, 23, 24):
+        P, _, w, _ = oracle.build_projection(oracle.autocorr_sum(X), n, L)
+        mse = oracle.projection_mse(X, P)
+        tail = float(np.sum(w[L:]))
+        assert abs(mse - tail) <= 1e-10 * float(np.sum(w)) + 1e-10 * tail
+
+
+def test_theorem1_top_eigenvectors_minimize_mse():
+    X = _calib(seed=7)
+    n, K = X.shape
+    L = 6
+    S = oracle.autocorr_sum(X)
+    P, _, w, _ = oracle.build_projection(S, n, L)
+    best = oracle.projection_mse(X, P)
+    r = rng(8)
+    for _ in range(100):
+        Q = synth.haar_orthonormal(r, K, L)
+        assert best <= oracle.projection_mse(X, Q) * (1 + 1e-12)
+    _, V, _ = oracle.eigh(S / n)
+    for _ in range(20):
+        idx = np.sort(r.choice(K, size=L, replace=False))
+        if np.array_equal(idx, np.arange(L)):
+            continue
+        assert best <= oracle.projection_mse(X, V[:, idx]) * (1 + 1e-12)
+
+
+def test_projection_columns_orthonormal_and_signs_normalized():
+    X = _calib(seed=9)
+    P, P_b, _, _ = oracle.build_projection(oracle.autocorr_sum(X), X.shape[0], 10)
+    assert np.allclose(P.T @ P, np.eye(10), atol=1e-12)
+    for j in range(10):
+        i = int(np.argmax(np.abs(P[:, j])))
+        assert P[i, j] > 0
+    assert np.array_equal(P_b, oracle.bf16_round(P))
+
+
+def test_prop1_bounds_hold_per_sample():
+    X = _calib(K=20, n=500, seed=10)
+    P, _, _, _ = oracle.build_projection(oracle.autocorr_sum(X), X.shape[0], 7)
+    Xt = oracle.reconstruct(X, P)
+    assert np.all(np.sum(Xt * Xt, 1) <= np.sum(X * X, 1) * (1 + 1e-12))
+    w = rng(11).standard_normal(20)
+    y, yt = X @ w, Xt @ w
+    bound = 2 * (w @ w) * np.sum(X * X, 1) - 2 * y * yt
+    assert np.all((y - yt) ** 2 <= bound + 1e-9 * np.abs(bound).max())
+
+
+# ---------------------------------------------------------------- Eq. 1 and Eq. 3
+
+def test_fold_project_contract_dense_brute_force():
+    r = rng(12)
+    N, K, M, L = 4, 6, 5, 3
+    X, W, P = r.standard_normal((N, K)), r.standard_normal((M, K)), r.standard_normal((K, L))
+    Wf = oracle.fold(P, W, round_bf16=False)
+    Z = oracle.project(X, P, round_bf16=False)
+    Y = oracle.contract(Z, Wf)
+    Yd = oracle.dense(X, W)
+    for l in range(L):
+        for m in range(M):
+            assert abs(Wf[l, m] - sum(P[k][l] * W[m][k] for k in range(K))) < 1e-13
+    for t in range(N):
+        for l in range(L):
+            assert abs(Z[t, l] - sum(X[t][k] * P[k][l] for k in range(K))) < 1e-13
+        for m in range(M):
+            assert abs(Y[t, m] - sum(Z[t][l] * Wf[l][m] for l in range(L))) < 1e-12
+            assert abs(Yd[t, m] - sum(W[m][k] * X[t][k] for k in range(K))) < 1e-13
+
+
+def test_eq3_associativity():
+    """(P^T W)^T (P^T X) = W^T (P P^T X) for non-square shapes."""
+    r = rng(13)
+    N, K, M, L = 9, 14, 11, 5
+    X, W = r.standard_normal((N, K)), r.standard_normal((M, K))
+    P = synth.haar_orthonormal(r, K, L)
+    Y, _, _ = oracle.forward(X, P, W, round_bf16=False)
+    assert np.allclose(Y, oracle.dense(oracle.reconstruct(X, P), W), rtol=1e-12, atol=1e-12)
+
+
+def test_full_rank_projection_is_exact():
+    """L = K gives P P^T = I, so the projected layer equals the dense one."""
+    X = _calib(K=16, n=40, seed=14)
+    W = rng(15).standard_normal((21, 16))
+    P, P_b, _, _ = oracle.build_projection(oracle.autocorr_sum(X), X.shape[0], 16)
+    Y, _, _ = oracle.forward(X, P, W, round_bf16=False)
+    Yd = oracle.dense(X, W)
+    assert np.allclose(Y, Yd, rtol=1e-12, atol=1e-12 * np.abs(Yd).max())
+    # with the bf16 projection and bf16 intermediates it still holds to bf16 accuracy
+    Yb, _, _ = oracle.forward(X, P_b, W)
+    assert np.linalg.norm(Yb - Yd) / np.linalg.norm(Yd) < 2e-2
+
+
+def test_rounded_intermediates_are_bf16_values():
+    r = rng(16)
+    X, W, P = r.standard_normal((8, 32)), r.standard_normal((24, 32)), r.standard_normal((32, 16))
+    Y, Z, Wf = oracle.forward(X, P, W)
+    assert np.array_equal(Z, oracle.bf16_round(Z))
+    assert np.array_equal(Wf, oracle.bf16_round(Wf))
+    assert np.array_equal(Z, oracle.bf16_round(oracle.project(X, P, round_bf16=False)))
