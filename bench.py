@@ -1,0 +1,397 @@
+"""Benchmark of the ESPACE projected linear layer on GB300 (one JSON line on rank 0).
+
+Workload (the metric's configuration): the Llama2-7B-shaped fused QKV projection at prefill,
+K = 4096 in-features, M = 12288 out-features, rank L = 2048 (50 % of K), N = 4096 tokens,
+bf16 inputs, fp32 accumulation, with synthetic activations (power-law spectrum i^-0.8,
+1 % outlier channels x20, log-normal channel scales) and W ~ N(0, 1/K).
+
+A step is one espace_linear_forward over the N-token batch: the rank-L projection
+Z = bf16(X P) and the folded product Y = Z W' (Eq. 3). Steps rotate over four independent
+(X, P, W') sets, 392 MB in all, so that no step finds its inputs in the 129 MB L2.
+value = algorithmic TFLOP/s, 2 N (K L + L M) per step, over the K timed steps (max over
+ranks). In the same run, and reported beside it in "rows": the dense W^T X baseline on the
+same tensor-core kernel (speedup = dense time / ESPACE time), the calibration accumulate
+(tcgen05 SYRK, Eq. 4) over 65,536 tokens, and the decode-shaped small-N forward at N = 1.
+
+--impl reference times the fp64 CPU oracle (the only reference this method has: the paper
+publishes no code) on a bounded sample of the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+import synth  # noqa: E402
+
+CONFIG = "llama2_qkv_prefill"
+METRIC = "ESPACE linear forward TFLOP/s (Llama2-7B QKV prefill, L=K/2)"
+UNIT = "TFLOP/s"
+SETS = 4
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-rows", action="store_true", help="skip the side measurements")
+    return ap.parse_args()
+
+
+def dist_init(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        torch.distributed.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d.get("bf16_tflops", 1900.0), d.get("bf16_tflops_sustained", 1700.0), d.get("hbm_gbs", 6800.0), "measured"
+    return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the GPU works."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.proc = None
+        self.device_index = device_index
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.device_index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        maxc = max(r[1] for r in rows)
+        loaded = [r for r in rows if r[0] > 0.5 * maxc] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in loaded for i, v in enumerate(r[2]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in loaded), "sm_max_mhz": maxc,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def cuda_events(n):
+    return [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+def run_reference(args, world, rank):
+    """fp64 oracle on the host cores, on a bounded sample of the workload."""
+    import oracle
+    if rank != 0:
+        return
+    cfg = synth.CONFIGS[CONFIG]
+    K, M, L = cfg["K"], cfg["M"], cfg["L"]
+    seed = synth.config_seed(CONFIG)
+    sample_tokens = 8
+    model = synth.ActivationModel(K, seed=seed)
+    X = synth.bf16_to_f64(model.sample(sample_tokens))
+    W = synth.bf16_to_f64(synth.weights(M, K, seed=seed))
+    Pb = oracle.bf16_round(synth.random_projection(K, L, seed=seed))
+    # W' = P^T W is folded offline (Sec. 2.2); it is an input of the timed forward here
+    Wf = oracle.bf16_round(Pb.T @ W.T)
+    flops_per_token = 2.0 * (K * L + L * M)
+    times = []
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        Z = oracle.project(X, Pb)
+        oracle.contract(Z, Wf)
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.append(dt)
+    total = sum(times)
+    value = flops_per_token * sample_tokens * len(times) / total / 1e12
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    sample = f"{sample_tokens} tokens of N={cfg['N']} per step (projection + folded product, fold precomputed)"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": "llama2_7b_qkv_prefill", "K": K, "M": M, "L": L, "N": cfg["N"]},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": min(cores, sample_tokens),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def cpu_baseline_leg():
+    import oracle
+    cfg = synth.CONFIGS[CONFIG]
+    K, M, L = cfg["K"], cfg["M"], cfg["L"]
+    seed = synth.config_seed(CONFIG)
+    sample_tokens = 8
+    model = synth.ActivationModel(K, seed=seed)
+    X = synth.bf16_to_f64(model.sample(sample_tokens))
+    W = synth.bf16_to_f64(synth.weights(M, K, seed=seed))
+    Pb = oracle.bf16_round(synth.random_projection(K, L, seed=seed))
+    Wf = oracle.bf16_round(Pb.T @ W.T)
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        oracle.contract(oracle.project(X, Pb), Wf)
+        reps += 1
+        if time.perf_counter() - t0 > 10.0 or reps >= 20:
+            break
+    dt = time.perf_counter() - t0
+    value = 2.0 * (K * L + L * M) * sample_tokens * reps / dt / 1e12
+    cores = min(os.cpu_count() or 1, sample_tokens)
+    return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{sample_tokens} tokens x {reps} repetitions of the fp64 oracle forward "
+                      f"(projection + folded product) at K={K}, L={L}, M={M}"}
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def run_ours(args, world, rank, local):
+    import paper_2410_05437_gb300 as esp
+    torch.cuda.set_device(local)
+    cfg = synth.CONFIGS[CONFIG]
+    K, M, L, N = cfg["K"], cfg["M"], cfg["L"], cfg["N"]
+    seed = synth.config_seed(CONFIG) + 1000 * rank
+    peak_tc, peak_tc_sus, peak_hbm, peak_kind = load_peaks()
+
+    model = synth.ActivationModel(K, seed=seed)
+    sets = []
+    for s in range(SETS):
+        X = model.sample_device(N, chunk=s)
+        W = synth.weights_device(M, K, seed=seed, chunk=s)
+        P = synth.random_projection(K, L, seed=seed + s)
+        p = esp.espace_proj_from_host(P, W)
+        sets.append({"X": X, "W": W, "p": p, "Y": torch.empty((N, M), dtype=torch.bfloat16, device="cuda")})
+    torch.cuda.synchronize()
+
+    flops = 2.0 * N * (K * L + L * M)
+    flops_phase2 = 2.0 * N * L * M
+    dense_flops = 2.0 * N * K * M
+
+    sampler = ClockSampler(local)
+    sampler.start()
+
+    # ---- warm-up
+    for i in range(args.warmup):
+        s = sets[i % SETS]
+        esp.espace_linear_forward(s["p"], s["X"], s["Y"])
+    torch.cuda.synchronize()
+
+    # ---- timed region: exactly K steps
+    starts, mids, ends = cuda_events(args.steps), cuda_events(args.steps), cuda_events(args.steps)
+    for e in mids:
+        e.record()                       # materialize the event handles
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    t_begin, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_begin.record()
+    for i in range(args.steps):
+        s = sets[i % SETS]
+        starts[i].record()
+        esp.espace_set_phase_event(mids[i])
+        esp.espace_linear_forward(s["p"], s["X"], s["Y"])
+        ends[i].record()
+    t_end.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    total_ms = max_over_ranks(t_begin.elapsed_time(t_end), world)
+    phase1 = [starts[i].elapsed_time(mids[i]) for i in range(args.steps)]
+    phase2 = [mids[i].elapsed_time(ends[i]) for i in range(args.steps)]
+    ms_per_step = total_ms / args.steps
+    value = flops * args.steps * world / (total_ms * 1e-3) / 1e12
+    esp.espace_check()
+
+    # ---- end to end through the C ABI with host buffers (pinned), copies inside the timed region
+    Xh = [s["X"].cpu().pin_memory() for s in sets]
+    Yh = torch.empty((N, M), dtype=torch.bfloat16).pin_memory()
+    Xd = torch.empty((N, K), dtype=torch.bfloat16, device="cuda")
+    e2e_steps = max(3, min(args.steps, 20))
+    for i in range(2):
+        Xd.copy_(Xh[i % SETS], non_blocking=True)
+        esp.espace_linear_forward(sets[i % SETS]["p"], Xd, sets[i % SETS]["Y"])
+        Yh.copy_(sets[i % SETS]["Y"], non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for i in range(e2e_steps):
+        s = sets[i % SETS]
+        Xd.copy_(Xh[i % SETS], non_blocking=True)
+        esp.espace_linear_forward(s["p"], Xd, s["Y"])
+        Yh.copy_(s["Y"], non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world) / e2e_steps
+    e2e_value = flops * world / (e2e_ms * 1e-3) / 1e12
+
+    rows = {}
+    if not args.no_rows:
+        rows = side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, ms_per_step)
+    clocks = sampler.stop()
+
+    p2_ms = statistics.mean(phase2)
+    achieved = flops_phase2 / (p2_ms * 1e-3) / 1e12
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded power-law activations with outlier channels; random-init W; random orthonormal P)",
+        "config": {"workload": "llama2_7b_qkv_prefill", "K": K, "M": M, "L": L, "N": N,
+                   "tokens_per_step_per_gpu": N, "parallelism": f"replicas{world}",
+                   "l2": f"inputs rotate over {SETS} sets of X, P, W' ({SETS * 2 * (N * K + K * L + L * M) / 1e6:.0f} MB > 129 MB L2)"},
+        "roofline": {"kernel": "tc_gemm_kernel (phase 2: Y = Z W')", "bound": "tensor",
+                     "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
+                     "frac": achieved / peak_tc, "peak_kind": f"{peak_kind} bf16 burst",
+                     "flops_per_launch": flops_phase2, "ms_per_launch": p2_ms, "traffic": None},
+        "phases_ms": {"project_XP": statistics.mean(phase1), "contract_ZW": p2_ms},
+        "roofline_step": {"frac_of_tensor_peak": (flops / (ms_per_step * 1e-3) / 1e12) / peak_tc,
+                          "roofline_ms": max(flops / (peak_tc * 1e12),
+                                             2.0 * (N * K + K * L + L * M + N * M) / (peak_hbm * 1e9)) * 1e3},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": N * K * 2,
+                "d2h_bytes_per_step": N * M * 2, "ms_per_step": e2e_ms},
+        "gpu_launches": 2 * args.steps,
+        "rows": rows,
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1:
+        try:
+            line["cpu_baseline"] = cpu_baseline_leg()
+        except Exception as ex:   # the baseline must not sink the GPU line
+            line["cpu_baseline"] = {"error": repr(ex)}
+    for s in sets:
+        esp.espace_proj_destroy(s["p"])
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, espace_ms):
+    rows = {}
+    reps = max(10, args.steps)
+    # dense baseline Y = X W^T on the same kernel
+    for i in range(3):
+        s = sets[i % SETS]
+        esp.espace_dense_forward(s["X"], s["W"], s["Y"])
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for i in range(reps):
+        s = sets[i % SETS]
+        esp.espace_dense_forward(s["X"], s["W"], s["Y"])
+    b.record()
+    torch.cuda.synchronize()
+    dense_ms = a.elapsed_time(b) / reps
+    dflops = 2.0 * N * K * M
+    rows["dense_forward"] = {"ms": dense_ms, "tflops": dflops / dense_ms / 1e9,
+                             "frac_tensor_peak": dflops / dense_ms / 1e9 / peak_tc,
+                             "speedup_espace_over_dense": dense_ms / espace_ms}
+    # calibration: S += X^T X over 65,536 tokens (tcgen05 SYRK)
+    n_cal = synth.CONFIGS[CONFIG]["calib_tokens"]
+    Xc = model.sample_device(n_cal, stream="calib_tokens")
+    h = esp.espace_calib_create(K)
+    esp.espace_calib_accumulate(h, Xc)
+    esp.espace_calib_reset(h)
+    torch.cuda.synchronize()
+    crep = 3
+    a.record()
+    for _ in range(crep):
+        esp.espace_calib_accumulate(h, Xc)
+    b.record()
+    torch.cuda.synchronize()
+    cal_ms = a.elapsed_time(b) / crep
+    cflops = float(n_cal) * K * (K + 1)
+    rows["calib_accumulate"] = {"tokens": n_cal, "ms": cal_ms, "tflops_symmetric": cflops / cal_ms / 1e9,
+                                "frac_tensor_peak": cflops / cal_ms / 1e9 / peak_tc}
+    esp.espace_calib_destroy(h)
+    del Xc
+    # decode-shaped forward at N = 1 (small-N streaming kernels)
+    x1 = [s["X"][:1].contiguous() for s in sets]
+    y1 = torch.empty((1, M), dtype=torch.bfloat16, device="cuda")
+    for i in range(3):
+        esp.espace_linear_forward(sets[i % SETS]["p"], x1[i % SETS], y1)
+    torch.cuda.synchronize()
+    drep = 200
+    a.record()
+    for i in range(drep):
+        esp.espace_linear_forward(sets[i % SETS]["p"], x1[i % SETS], y1)
+    b.record()
+    torch.cuda.synchronize()
+    d_ms = a.elapsed_time(b) / drep
+    Lp = (L + 63) // 64 * 64
+    dbytes = 2.0 * (K * Lp + Lp * M + K + M)
+    rows["decode_n1"] = {"us": d_ms * 1e3, "gbs": dbytes / d_ms / 1e6, "frac_hbm": dbytes / d_ms / 1e6 / peak_hbm}
+    return rows
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_init(args.gpus)
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_ours(args, world, rank, local)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

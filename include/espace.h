@@ -1,0 +1,206 @@
+/*
+ * espace.h -- C ABI of the GB300 (sm_103a) library for ESPACE's projected linear layer.
+ *
+ * ESPACE (arXiv 2410.05437) replaces a linear layer Y = W^T X (Sec. 2.1, Eq. 1) by
+ * Y = (P^T W)^T (P^T X) (Sec. 2.2, Eq. 3), where P (K x L) holds the L principal
+ * eigenvectors of the activation autocorrelation C = E[x x^T] (Sec. 3.1, Eq. 4, Thm. 1)
+ * and W' = P^T W is folded once before deployment (Sec. 2.2).
+ *
+ * Letters: K = input features, M = output features, N = tokens, L = rank (1 <= L <= K).
+ * Storage is row-major and token-major, as PyTorch keeps activations:
+ *   X  [N][K] bf16    input tokens, one per row
+ *   W  [M][K] bf16    dense weight in nn.Linear layout (row m = output feature m)
+ *   Y  [N][M] bf16    output tokens
+ * In this layout Eq. 3 reads Z[N][L] = X P and Y = Z W'.
+ *
+ * Conventions shared by every call:
+ *   - "bf16" buffers hold IEEE bfloat16 bit patterns (uint16_t); "_dev" pointers are CUDA
+ *     device pointers of the current device and must be 16-byte aligned; K must be a
+ *     multiple of 8 and M a multiple of 8 (16-byte row pitch, needed by the TMA engine).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Calls
+ *     marked "async" only enqueue work on it; the caller synchronizes before reading results.
+ *   - The caller owns X, W, Y and streams. The library owns handles and the device memory
+ *     behind them (S, P^T, W'^T, the Z scratch) and frees it in the *_destroy calls.
+ *   - Every int-returning call returns ESPACE_OK (0) or one of the ESPACE_ERR_* codes below;
+ *     nothing throws across the ABI, a rejected argument never launches a kernel, and
+ *     espace_last_error() describes the most recent failure of the calling thread.
+ *   - Device-side waits are bounded: a kernel that gives up records ESPACE_ERR_TIMEOUT in a
+ *     per-device status word, which espace_check() reports (and clears).
+ */
+#ifndef ESPACE_H
+#define ESPACE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ESPACE_OK            0
+#define ESPACE_ERR_ARG       1   /* null pointer or value out of range */
+#define ESPACE_ERR_SHAPE     2   /* sizes inconsistent with the handle or unsupported */
+#define ESPACE_ERR_ALIGN     3   /* pointer not 16-byte aligned */
+#define ESPACE_ERR_CUDA      4   /* a CUDA runtime / driver call failed */
+#define ESPACE_ERR_TIMEOUT   5   /* a device-side wait exceeded its limit */
+#define ESPACE_ERR_STATE     6   /* call not valid in the handle's state (e.g. no tokens) */
+#define ESPACE_ERR_NOMEM     7   /* device or host allocation failed */
+#define ESPACE_ERR_NUMERIC   8   /* the host eigen-solver did not converge */
+
+typedef struct espace_calib_s* espace_calib_t;   /* autocorrelation accumulator (Eq. 4)   */
+typedef struct espace_proj_s*  espace_proj_t;    /* calibrated P^T and folded W'^T (Eq. 3) */
+
+/* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
+int espace_version(void);
+
+/* Text for the calling thread's most recent failure ("" if none). Valid until the next
+ * failing call on the same thread. */
+const char* espace_last_error(void);
+
+/* ---------------------------------------------------------------------------------------
+ * Calibration (Sec. 3.1, Eq. 4): C = X X^T / n summed over calibration tokens. The paper
+ * averages per-batch means; the library keeps the running sum S and the token count n and
+ * forms C = S / n, which is the same estimate for equal-size batches and the token-weighted
+ * mean otherwise. No mean is subtracted (Sec. 3.2 omits input normalization).
+ * ------------------------------------------------------------------------------------- */
+
+/* Creates an accumulator for K-dimensional activations with S = 0, n = 0. Allocates an
+ * fp32 K x K device buffer. K: multiple of 8, 8 <= K <= 65536. */
+int espace_calib_create(int64_t K, espace_calib_t* out);
+
+/* Async. S += X^T X over the N rows of X_dev ([N][K] bf16) and n += N, on tcgen05 tensor
+ * cores with fp32 accumulation; only the upper triangle of S is stored. N = 0 is a no-op.
+ * The host-side counter n is updated when the call is enqueued. */
+int espace_calib_accumulate(espace_calib_t h, const void* X_dev, int64_t N, void* stream);
+
+/* Same, with each token first scaled to unit L2 norm (Cor. 1: the autocorrelation of
+ * x / ||x|| whose eigenvectors minimize the normalized MSE of Eq. 7). Tokens of zero norm
+ * add nothing but still count in n. Do not mix with espace_calib_accumulate on one handle. */
+int espace_calib_accumulate_normalized(espace_calib_t h, const void* X_dev, int64_t N,
+                                       void* stream);
+
+/* Synchronizes `stream`, then writes C = S / n as a full symmetric K x K fp64 matrix
+ * (C_host may be NULL) and the token count (n_out may be NULL). ESPACE_ERR_STATE if n = 0
+ * and C_host != NULL. */
+int espace_calib_read(espace_calib_t h, double* C_host, int64_t* n_out, void* stream);
+
+/* Checkpointing of the accumulator: export copies the raw upper-triangular fp32 sum S
+ * (K*K floats, row-major, lower triangle unspecified) and n to the host after synchronizing
+ * `stream`; import replaces them. Exported sums of several shards may be added and imported
+ * into one handle (the all-reduce step of data-parallel calibration). */
+int espace_calib_export(espace_calib_t h, float* S_host, int64_t* n_out, void* stream);
+int espace_calib_import(espace_calib_t h, const float* S_host, int64_t n, void* stream);
+
+/* Resets S = 0 and n = 0 (async on `stream`). */
+int espace_calib_reset(espace_calib_t h, void* stream);
+
+void espace_calib_destroy(espace_calib_t h);
+
+/* ---------------------------------------------------------------------------------------
+ * Projection and fold (Thm. 1, Sec. 2.2)
+ * ------------------------------------------------------------------------------------- */
+
+/* Synchronous. Builds the projected layer from a calibrated accumulator:
+ *   1. C = S / n in fp64 on the host;
+ *   2. symmetric eigen-decomposition of C in fp64 on the host (Householder
+ *      tridiagonalization and implicit QR), eigenvalues sorted decreasing (Sec. 3.1);
+ *   3. P = the first L eigenvectors (Thm. 1), each column's largest-magnitude entry made
+ *      positive (lowest index on ties), rounded to bf16;
+ *   4. W'^T = W P rounded to bf16, i.e. W' = P^T W (Sec. 2.2), on the GPU with fp32
+ *      accumulation, from W_dev ([M][K] bf16, read once; the caller may free it after).
+ * The handle keeps P^T as [Lp][K] and W'^T as [M][Lp] bf16 with L rounded up to Lp, a
+ * multiple of 64; the padding rows/columns are zero, which leaves Y unchanged. */
+int espace_build_projection(espace_calib_t h, const void* W_dev, int64_t M, int64_t L,
+                            void* stream, espace_proj_t* out);
+
+/* Synchronous. Same as steps 3 (rounding only) and 4 above for a given fp64 P_host
+ * ([K][L], row-major), with no eigen-solve: used to feed one projection to several
+ * implementations. */
+int espace_proj_from_host(int64_t K, int64_t M, int64_t L, const double* P_host,
+                          const void* W_dev, void* stream, espace_proj_t* out);
+
+/* Shape of a projection: any output pointer may be NULL. */
+int espace_proj_shape(espace_proj_t p, int64_t* K, int64_t* M, int64_t* L);
+
+/* The K eigenvalues of C in decreasing order (only for handles made by
+ * espace_build_projection; ESPACE_ERR_STATE otherwise). */
+int espace_proj_eigenvalues(espace_proj_t p, double* dst);
+
+/* Copies P as bf16 [K][L] (row-major) to the host. */
+int espace_proj_read_P(espace_proj_t p, uint16_t* P_host);
+
+/* Copies W' as bf16 [L][M] (row-major) to the host. */
+int espace_proj_read_Wfold(espace_proj_t p, uint16_t* Wf_host);
+
+/* Checkpointing of a projection: export writes P^T [Lp][K] and W'^T [M][Lp] bf16 and the
+ * K eigenvalues (zeros if unknown) to host buffers sized from espace_proj_shape (Lp = L
+ * rounded up to a multiple of 64); import rebuilds a handle from them. */
+int espace_proj_export(espace_proj_t p, uint16_t* PT_host, uint16_t* WfT_host, double* evals);
+int espace_proj_import(int64_t K, int64_t M, int64_t L, const uint16_t* PT_host,
+                       const uint16_t* WfT_host, const double* evals, espace_proj_t* out);
+
+void espace_proj_destroy(espace_proj_t p);
+
+/* ---------------------------------------------------------------------------------------
+ * Forward (Sec. 2.2, Eq. 3)
+ * ------------------------------------------------------------------------------------- */
+
+/* Async. Y = (P^T W)^T (P^T X) for the N tokens of X_dev ([N][K] bf16) into Y_dev
+ * ([N][M] bf16): Z = X P is accumulated in fp32 and rounded to bf16 (the paper computes in
+ * BF16, Sec. A.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. Small N runs
+ * a bandwidth-bound kernel that streams P and W' once; larger N runs the tcgen05
+ * tensor-core path. N = 0 is a no-op. The first call with a larger N than any before on
+ * this handle allocates the Z scratch (synchronously); later calls allocate nothing. */
+int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev,
+                          void* stream);
+
+/* As espace_linear_forward with the kernel family chosen by the caller:
+ * path 0 = automatic, 1 = tensor-core kernels, 2 = small-N streaming kernels
+ * (ESPACE_ERR_SHAPE if N or the layer is too large for the small-N kernels). */
+#define ESPACE_PATH_AUTO    0
+#define ESPACE_PATH_TENSOR  1
+#define ESPACE_PATH_SMALL_N 2
+int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev,
+                               void* stream, int path);
+
+/* Async. The uncompressed layer of Eq. 1, Y = W^T X, as Y_dev[N][M] = X_dev[N][K] W_dev^T
+ * with W_dev in [M][K] layout, on the same tcgen05 kernel with fp32 accumulation and bf16
+ * output: the baseline the projected layer is measured against. */
+int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev,
+                         int64_t M, void* Y_dev, void* stream);
+
+/* Synchronizes `stream` and reports (then clears) the device status word: ESPACE_OK, or
+ * ESPACE_ERR_TIMEOUT if a kernel gave up waiting since the last check, or ESPACE_ERR_CUDA
+ * if the stream reported an error. */
+int espace_check(void* stream);
+
+/* Measurement hook: the next espace_linear_forward / espace_linear_forward_path call on
+ * this thread records `event` (a cudaEvent_t) on its stream between the rank-L projection
+ * kernel (Z = X P) and the folded-weight kernel (Y = Z W'), so that the two products of
+ * Eq. 3 can be timed separately. One-shot: cleared by that call. NULL cancels. */
+int espace_set_phase_event(void* event);
+
+/* Test hook: upper bound in nanoseconds for every device-side wait of later launches
+ * (default 4e9). 0 restores the default. */
+int espace_set_wait_limit_ns(uint64_t ns);
+
+/* Test hook for the bounded waits: launches (async) one thread that waits on a barrier
+ * nothing completes, gives up after limit_ns (at most 1e9) and records ESPACE_ERR_TIMEOUT,
+ * so that the next espace_check() reports it. Nothing faults and the context stays usable. */
+int espace_debug_wait_timeout(uint64_t limit_ns, void* stream);
+
+/* ---------------------------------------------------------------------------------------
+ * Host-only helper (no GPU needed)
+ * ------------------------------------------------------------------------------------- */
+
+/* fp64 symmetric eigen-decomposition used by espace_build_projection: A_host is K x K
+ * row-major symmetric (only read); w receives the eigenvalues in decreasing order and V
+ * (K x K row-major, may be NULL) the unit eigenvectors as columns, with the sign
+ * convention of espace_build_projection. ESPACE_ERR_NUMERIC if the QR iteration does not
+ * converge. Uses up to `threads` host threads (0 = all cores). */
+int espace_host_eigh(const double* A_host, int64_t K, double* w, double* V, int threads);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ESPACE_H */

@@ -1,0 +1,645 @@
+// espace_api.cu -- the C ABI declared in include/espace.h: argument checks, handles and
+// their device memory, the host side of calibration and projection building, and dispatch
+// of the forward pass to the tcgen05 or the streaming kernels.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <atomic>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/espace.h"
+#include "kernels.h"
+
+namespace espace {
+int host_eigh(const double* A, int64_t n, double* w, double* V, int threads);
+}
+
+using namespace espace;
+
+// ============================================================================ errors
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const char* fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return code;
+}
+
+int fail_cuda(cudaError_t e, const char* what)
+{
+    return fail(ESPACE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define CUDA_TRY(expr, what)                        \
+    do {                                            \
+        cudaError_t _e = (expr);                    \
+        if (_e != cudaSuccess) return fail_cuda(_e, what); \
+    } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+std::atomic<uint64_t> g_wait_limit_ns{4000000000ull};
+thread_local cudaEvent_t g_phase_event = nullptr;
+
+// Makes `device` current for the lifetime of the guard.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int device)
+    {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (device >= 0 && device != prev) ok = cudaSetDevice(device) == cudaSuccess;
+    }
+    ~DeviceGuard()
+    {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+// bf16 bits of the value nearest to x, ties to even, in one rounding from fp64: x is first
+// narrowed to fp32 with rounding to odd, which keeps the later fp32 -> bf16 rounding to
+// nearest correct (Boldo & Melquiond, "Emulation of FMA and correctly rounded sums: proved
+// algorithms using rounding to odd", IEEE TC 2008).
+uint16_t bf16_from_double(double x)
+{
+    if (x != x) return 0x7fc0;
+    float f = static_cast<float>(x);
+    if (static_cast<double>(f) != x && !__builtin_isinf(f)) {
+        // truncate towards zero, then force the last bit to one (round to odd)
+        if (fabs(static_cast<double>(f)) > fabs(x)) f = nextafterf(f, 0.0f);
+        uint32_t b;
+        memcpy(&b, &f, 4);
+        b |= 1u;
+        memcpy(&f, &b, 4);
+    }
+    uint32_t b;
+    memcpy(&b, &f, 4);
+    if ((b & 0x7f800000u) == 0x7f800000u) return static_cast<uint16_t>(b >> 16);   // inf
+    b += 0x7fffu + ((b >> 16) & 1u);
+    return static_cast<uint16_t>(b >> 16);
+}
+
+int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+}  // namespace
+
+// ============================================================================ device state
+
+namespace espace {
+
+int device_info(DeviceInfo** out)
+{
+    static std::mutex mu;
+    static std::vector<DeviceInfo*> infos;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+    std::lock_guard<std::mutex> lock(mu);
+    if (dev >= static_cast<int>(infos.size())) infos.resize(dev + 1, nullptr);
+    if (infos[dev] == nullptr) {
+        DeviceInfo* d = new DeviceInfo();
+        d->device = dev;
+        e = cudaDeviceGetAttribute(&d->num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) {
+            delete d;
+            return fail_cuda(e, "cudaDeviceGetAttribute");
+        }
+        int major = 0, minor = 0;
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+        if (major != 10 || minor != 3) {
+            delete d;
+            return fail(ESPACE_ERR_STATE,
+                        "device %d is sm_%d%d; this library is built for sm_103a only", dev,
+                        major, minor);
+        }
+        e = cudaMalloc(&d->status, sizeof(int));
+        if (e != cudaSuccess) {
+            delete d;
+            return fail_cuda(e, "cudaMalloc(status)");
+        }
+        e = cudaMemset(d->status, 0, sizeof(int));
+        if (e != cudaSuccess) {
+            cudaFree(d->status);
+            delete d;
+            return fail_cuda(e, "cudaMemset(status)");
+        }
+        infos[dev] = d;
+    }
+    *out = infos[dev];
+    return ESPACE_OK;
+}
+
+uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
+
+}  // namespace espace
+
+// ============================================================================ handles
+
+struct espace_calib_s {
+    int64_t K = 0;
+    int device = 0;
+    float* S = nullptr;            // [K][K] fp32, upper triangle valid
+    int64_t n = 0;
+    int mode = 0;                  // 0 unset, 1 plain, 2 normalized (Cor. 1)
+    void* xn = nullptr;            // scratch for normalized tokens
+    int64_t xn_tokens = 0;
+};
+
+struct espace_proj_s {
+    int64_t K = 0, M = 0, L = 0, Lp = 0;
+    int device = 0;
+    uint16_t* PT = nullptr;        // [Lp][K] bf16, rows >= L zero
+    uint16_t* WfT = nullptr;       // [M][Lp] bf16, columns >= L zero
+    std::vector<double> evals;     // K eigenvalues, decreasing (if calibrated)
+    uint16_t* Z = nullptr;         // [zcap][Lp] bf16 scratch for the rank-L intermediate
+    int64_t zcap = 0;
+    std::mutex mu;                 // guards Z growth
+};
+
+extern "C" {
+
+int espace_version(void) { return 100; }
+
+const char* espace_last_error(void) { return g_last_error.c_str(); }
+
+int espace_set_phase_event(void* event)
+{
+    g_phase_event = static_cast<cudaEvent_t>(event);
+    return ESPACE_OK;
+}
+
+int espace_set_wait_limit_ns(uint64_t ns)
+{
+    g_wait_limit_ns.store(ns == 0 ? 4000000000ull : ns);
+    return ESPACE_OK;
+}
+
+int espace_host_eigh(const double* A_host, int64_t K, double* w, double* V, int threads)
+{
+    if (A_host == nullptr || w == nullptr) return fail(ESPACE_ERR_ARG, "espace_host_eigh: null pointer");
+    if (K < 1 || K > 65536) return fail(ESPACE_ERR_SHAPE, "espace_host_eigh: K=%lld out of range", (long long)K);
+    const int rc = host_eigh(A_host, K, w, V, threads);
+    if (rc != ESPACE_OK) return fail(rc, "espace_host_eigh: QR iteration did not converge");
+    return ESPACE_OK;
+}
+
+// ---------------------------------------------------------------------------- calibration
+
+int espace_calib_create(int64_t K, espace_calib_t* out)
+{
+    if (out == nullptr) return fail(ESPACE_ERR_ARG, "espace_calib_create: out is null");
+    *out = nullptr;
+    if (K < 8 || K > 65536 || K % 8 != 0)
+        return fail(ESPACE_ERR_SHAPE, "espace_calib_create: K=%lld must be a multiple of 8 in [8, 65536]", (long long)K);
+    DeviceInfo* dev = nullptr;
+    int rc = device_info(&dev);
+    if (rc != ESPACE_OK) return rc;
+    espace_calib_s* h = new espace_calib_s();
+    h->K = K;
+    h->device = dev->device;
+    cudaError_t e = cudaMalloc(&h->S, sizeof(float) * K * K);
+    if (e != cudaSuccess) {
+        delete h;
+        return fail(ESPACE_ERR_NOMEM, "espace_calib_create: cudaMalloc of %lld bytes: %s",
+                    (long long)(sizeof(float) * K * K), cudaGetErrorString(e));
+    }
+    e = cudaMemset(h->S, 0, sizeof(float) * K * K);
+    if (e != cudaSuccess) {
+        cudaFree(h->S);
+        delete h;
+        return fail_cuda(e, "espace_calib_create: cudaMemset");
+    }
+    *out = h;
+    return ESPACE_OK;
+}
+
+static int calib_accumulate_impl(espace_calib_t h, const void* X, int64_t N, void* stream,
+                                 int mode)
+{
+    if (h == nullptr) return fail(ESPACE_ERR_ARG, "calib_accumulate: null handle");
+    if (N < 0) return fail(ESPACE_ERR_SHAPE, "calib_accumulate: N=%lld < 0", (long long)N);
+    if (N == 0) return ESPACE_OK;
+    if (X == nullptr) return fail(ESPACE_ERR_ARG, "calib_accumulate: X is null");
+    if (!aligned16(X)) return fail(ESPACE_ERR_ALIGN, "calib_accumulate: X not 16-byte aligned");
+    if (N > (int64_t(1) << 31) - 64) return fail(ESPACE_ERR_SHAPE, "calib_accumulate: N=%lld too large for one call", (long long)N);
+    if (h->mode != 0 && h->mode != mode)
+        return fail(ESPACE_ERR_STATE, "calib_accumulate: plain and normalized accumulation mixed on one handle");
+    DeviceGuard g(h->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const void* src = X;
+    if (mode == 2) {
+        if (h->xn_tokens < N) {
+            CUDA_TRY(cudaStreamSynchronize(st), "calib_accumulate_normalized: sync");
+            if (h->xn) cudaFree(h->xn);
+            h->xn = nullptr;
+            h->xn_tokens = 0;
+            cudaError_t e = cudaMalloc(&h->xn, sizeof(uint16_t) * N * h->K);
+            if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "calib_accumulate_normalized: scratch: %s", cudaGetErrorString(e));
+            h->xn_tokens = N;
+        }
+        CUDA_TRY(launch_normalize_rows(X, N, static_cast<int>(h->K), h->xn, st), "normalize_rows launch");
+        src = h->xn;
+    }
+    CUDA_TRY(launch_syrk_upper(src, N, static_cast<int>(h->K), h->S, st), "syrk launch");
+    h->mode = mode;
+    h->n += N;
+    return ESPACE_OK;
+}
+
+int espace_calib_accumulate(espace_calib_t h, const void* X_dev, int64_t N, void* stream)
+{
+    return calib_accumulate_impl(h, X_dev, N, stream, 1);
+}
+
+int espace_calib_accumulate_normalized(espace_calib_t h, const void* X_dev, int64_t N, void* stream)
+{
+    return calib_accumulate_impl(h, X_dev, N, stream, 2);
+}
+
+static int read_sum(espace_calib_t h, std::vector<float>& S, void* stream)
+{
+    DeviceGuard g(h->device);
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "calib read: sync");
+    S.resize(static_cast<size_t>(h->K * h->K));
+    CUDA_TRY(cudaMemcpy(S.data(), h->S, sizeof(float) * S.size(), cudaMemcpyDeviceToHost), "calib read: copy");
+    return ESPACE_OK;
+}
+
+static void mirror_scaled(const std::vector<float>& S, int64_t K, double scale, double* C)
+{
+    for (int64_t i = 0; i < K; ++i)
+        for (int64_t j = 0; j < K; ++j) {
+            const int64_t a = std::min(i, j), b = std::max(i, j);
+            C[i * K + j] = static_cast<double>(S[a * K + b]) * scale;
+        }
+}
+
+int espace_calib_read(espace_calib_t h, double* C_host, int64_t* n_out, void* stream)
+{
+    if (h == nullptr) return fail(ESPACE_ERR_ARG, "espace_calib_read: null handle");
+    if (n_out) *n_out = h->n;
+    if (C_host == nullptr) {
+        DeviceGuard g(h->device);
+        CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "calib read: sync");
+        return ESPACE_OK;
+    }
+    if (h->n == 0) return fail(ESPACE_ERR_STATE, "espace_calib_read: no tokens accumulated");
+    std::vector<float> S;
+    int rc = read_sum(h, S, stream);
+    if (rc != ESPACE_OK) return rc;
+    mirror_scaled(S, h->K, 1.0 / static_cast<double>(h->n), C_host);
+    return ESPACE_OK;
+}
+
+int espace_calib_export(espace_calib_t h, float* S_host, int64_t* n_out, void* stream)
+{
+    if (h == nullptr || S_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_calib_export: null pointer");
+    std::vector<float> S;
+    int rc = read_sum(h, S, stream);
+    if (rc != ESPACE_OK) return rc;
+    memcpy(S_host, S.data(), sizeof(float) * S.size());
+    if (n_out) *n_out = h->n;
+    return ESPACE_OK;
+}
+
+int espace_calib_import(espace_calib_t h, const float* S_host, int64_t n, void* stream)
+{
+    if (h == nullptr || S_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_calib_import: null pointer");
+    if (n < 0) return fail(ESPACE_ERR_ARG, "espace_calib_import: n < 0");
+    DeviceGuard g(h->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    CUDA_TRY(cudaStreamSynchronize(st), "calib import: sync");
+    CUDA_TRY(cudaMemcpy(h->S, S_host, sizeof(float) * h->K * h->K, cudaMemcpyHostToDevice), "calib import: copy");
+    h->n = n;
+    return ESPACE_OK;
+}
+
+int espace_calib_reset(espace_calib_t h, void* stream)
+{
+    if (h == nullptr) return fail(ESPACE_ERR_ARG, "espace_calib_reset: null handle");
+    DeviceGuard g(h->device);
+    CUDA_TRY(launch_zero_f32(h->S, h->K * h->K, static_cast<cudaStream_t>(stream)), "calib reset");
+    h->n = 0;
+    h->mode = 0;
+    return ESPACE_OK;
+}
+
+void espace_calib_destroy(espace_calib_t h)
+{
+    if (h == nullptr) return;
+    DeviceGuard g(h->device);
+    cudaDeviceSynchronize();
+    if (h->S) cudaFree(h->S);
+    if (h->xn) cudaFree(h->xn);
+    delete h;
+}
+
+// ---------------------------------------------------------------------------- projection
+
+static int proj_create(int64_t K, int64_t M, int64_t L, espace_proj_s** out)
+{
+    DeviceInfo* dev = nullptr;
+    int rc = device_info(&dev);
+    if (rc != ESPACE_OK) return rc;
+    espace_proj_s* p = new espace_proj_s();
+    p->K = K;
+    p->M = M;
+    p->L = L;
+    p->Lp = round_up(L, 64);
+    p->device = dev->device;
+    cudaError_t e = cudaMalloc(&p->PT, sizeof(uint16_t) * p->Lp * K);
+    if (e == cudaSuccess) e = cudaMalloc(&p->WfT, sizeof(uint16_t) * M * p->Lp);
+    if (e != cudaSuccess) {
+        if (p->PT) cudaFree(p->PT);
+        delete p;
+        return fail(ESPACE_ERR_NOMEM, "projection: cudaMalloc: %s", cudaGetErrorString(e));
+    }
+    *out = p;
+    return ESPACE_OK;
+}
+
+static int check_proj_shape(int64_t K, int64_t M, int64_t L)
+{
+    if (K < 8 || K % 8 != 0 || K > 65536)
+        return fail(ESPACE_ERR_SHAPE, "K=%lld must be a multiple of 8 in [8, 65536]", (long long)K);
+    if (M < 8 || M % 8 != 0 || M > (int64_t(1) << 30))
+        return fail(ESPACE_ERR_SHAPE, "M=%lld must be a positive multiple of 8", (long long)M);
+    if (L < 1 || L > K) return fail(ESPACE_ERR_SHAPE, "L=%lld must be in [1, K=%lld]", (long long)L, (long long)K);
+    return ESPACE_OK;
+}
+
+// Uploads P (fp64 [K][L] row-major) as bf16 P^T [Lp][K] and folds W'^T = W P on the GPU.
+static int proj_upload_and_fold(espace_proj_s* p, const double* P, const void* W, cudaStream_t st)
+{
+    const int64_t K = p->K, L = p->L, Lp = p->Lp;
+    std::vector<uint16_t> pt(static_cast<size_t>(Lp * K), 0);
+    for (int64_t l = 0; l < L; ++l)
+        for (int64_t k = 0; k < K; ++k) pt[l * K + k] = bf16_from_double(P[k * L + l]);
+    CUDA_TRY(cudaStreamSynchronize(st), "projection: sync");
+    CUDA_TRY(cudaMemcpy(p->PT, pt.data(), sizeof(uint16_t) * pt.size(), cudaMemcpyHostToDevice), "projection: upload P");
+    CUDA_TRY(launch_gemm_tn(W, K, p->PT, K, static_cast<int>(p->M), static_cast<int>(Lp),
+                            static_cast<int>(K), p->WfT, Lp, st),
+             "projection: fold launch");
+    CUDA_TRY(cudaStreamSynchronize(st), "projection: fold");
+    return ESPACE_OK;
+}
+
+int espace_proj_from_host(int64_t K, int64_t M, int64_t L, const double* P_host, const void* W_dev,
+                          void* stream, espace_proj_t* out)
+{
+    if (out == nullptr || P_host == nullptr || W_dev == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_proj_from_host: null pointer");
+    *out = nullptr;
+    int rc = check_proj_shape(K, M, L);
+    if (rc != ESPACE_OK) return rc;
+    if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_proj_from_host: W not 16-byte aligned");
+    espace_proj_s* p = nullptr;
+    rc = proj_create(K, M, L, &p);
+    if (rc != ESPACE_OK) return rc;
+    rc = proj_upload_and_fold(p, P_host, W_dev, static_cast<cudaStream_t>(stream));
+    if (rc != ESPACE_OK) {
+        espace_proj_destroy(p);
+        return rc;
+    }
+    *out = p;
+    return ESPACE_OK;
+}
+
+int espace_build_projection(espace_calib_t h, const void* W_dev, int64_t M, int64_t L, void* stream,
+                            espace_proj_t* out)
+{
+    if (out == nullptr || h == nullptr || W_dev == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_build_projection: null pointer");
+    *out = nullptr;
+    const int64_t K = h->K;
+    int rc = check_proj_shape(K, M, L);
+    if (rc != ESPACE_OK) return rc;
+    if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_build_projection: W not 16-byte aligned");
+    if (h->n == 0) return fail(ESPACE_ERR_STATE, "espace_build_projection: no calibration tokens");
+    DeviceGuard g(h->device);
+    std::vector<float> S;
+    rc = read_sum(h, S, stream);
+    if (rc != ESPACE_OK) return rc;
+    std::vector<double> C(static_cast<size_t>(K * K)), w(K), V(static_cast<size_t>(K * K));
+    mirror_scaled(S, K, 1.0 / static_cast<double>(h->n), C.data());
+    rc = host_eigh(C.data(), K, w.data(), V.data(), 0);
+    if (rc != ESPACE_OK) return fail(rc, "espace_build_projection: eigen-solver did not converge");
+    std::vector<double> P(static_cast<size_t>(K * L));
+    for (int64_t k = 0; k < K; ++k)
+        for (int64_t l = 0; l < L; ++l) P[k * L + l] = V[k * K + l];
+    espace_proj_s* p = nullptr;
+    rc = proj_create(K, M, L, &p);
+    if (rc != ESPACE_OK) return rc;
+    p->evals = w;
+    rc = proj_upload_and_fold(p, P.data(), W_dev, static_cast<cudaStream_t>(stream));
+    if (rc != ESPACE_OK) {
+        espace_proj_destroy(p);
+        return rc;
+    }
+    *out = p;
+    return ESPACE_OK;
+}
+
+int espace_proj_shape(espace_proj_t p, int64_t* K, int64_t* M, int64_t* L)
+{
+    if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_shape: null handle");
+    if (K) *K = p->K;
+    if (M) *M = p->M;
+    if (L) *L = p->L;
+    return ESPACE_OK;
+}
+
+int espace_proj_eigenvalues(espace_proj_t p, double* dst)
+{
+    if (p == nullptr || dst == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_eigenvalues: null pointer");
+    if (p->evals.empty()) return fail(ESPACE_ERR_STATE, "espace_proj_eigenvalues: projection was not calibrated");
+    memcpy(dst, p->evals.data(), sizeof(double) * p->evals.size());
+    return ESPACE_OK;
+}
+
+int espace_proj_read_P(espace_proj_t p, uint16_t* P_host)
+{
+    if (p == nullptr || P_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_read_P: null pointer");
+    DeviceGuard g(p->device);
+    std::vector<uint16_t> pt(static_cast<size_t>(p->Lp * p->K));
+    CUDA_TRY(cudaDeviceSynchronize(), "read_P: sync");
+    CUDA_TRY(cudaMemcpy(pt.data(), p->PT, sizeof(uint16_t) * pt.size(), cudaMemcpyDeviceToHost), "read_P: copy");
+    for (int64_t k = 0; k < p->K; ++k)
+        for (int64_t l = 0; l < p->L; ++l) P_host[k * p->L + l] = pt[l * p->K + k];
+    return ESPACE_OK;
+}
+
+int espace_proj_read_Wfold(espace_proj_t p, uint16_t* Wf_host)
+{
+    if (p == nullptr || Wf_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_read_Wfold: null pointer");
+    DeviceGuard g(p->device);
+    std::vector<uint16_t> wt(static_cast<size_t>(p->M * p->Lp));
+    CUDA_TRY(cudaDeviceSynchronize(), "read_Wfold: sync");
+    CUDA_TRY(cudaMemcpy(wt.data(), p->WfT, sizeof(uint16_t) * wt.size(), cudaMemcpyDeviceToHost), "read_Wfold: copy");
+    for (int64_t l = 0; l < p->L; ++l)
+        for (int64_t m = 0; m < p->M; ++m) Wf_host[l * p->M + m] = wt[m * p->Lp + l];
+    return ESPACE_OK;
+}
+
+int espace_proj_export(espace_proj_t p, uint16_t* PT_host, uint16_t* WfT_host, double* evals)
+{
+    if (p == nullptr || PT_host == nullptr || WfT_host == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_proj_export: null pointer");
+    DeviceGuard g(p->device);
+    CUDA_TRY(cudaDeviceSynchronize(), "proj_export: sync");
+    CUDA_TRY(cudaMemcpy(PT_host, p->PT, sizeof(uint16_t) * p->Lp * p->K, cudaMemcpyDeviceToHost), "proj_export: P");
+    CUDA_TRY(cudaMemcpy(WfT_host, p->WfT, sizeof(uint16_t) * p->M * p->Lp, cudaMemcpyDeviceToHost), "proj_export: W'");
+    if (evals) {
+        for (int64_t i = 0; i < p->K; ++i) evals[i] = p->evals.empty() ? 0.0 : p->evals[i];
+    }
+    return ESPACE_OK;
+}
+
+int espace_proj_import(int64_t K, int64_t M, int64_t L, const uint16_t* PT_host, const uint16_t* WfT_host,
+                       const double* evals, espace_proj_t* out)
+{
+    if (out == nullptr || PT_host == nullptr || WfT_host == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_proj_import: null pointer");
+    *out = nullptr;
+    int rc = check_proj_shape(K, M, L);
+    if (rc != ESPACE_OK) return rc;
+    espace_proj_s* p = nullptr;
+    rc = proj_create(K, M, L, &p);
+    if (rc != ESPACE_OK) return rc;
+    cudaError_t e = cudaMemcpy(p->PT, PT_host, sizeof(uint16_t) * p->Lp * K, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(p->WfT, WfT_host, sizeof(uint16_t) * M * p->Lp, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        espace_proj_destroy(p);
+        return fail_cuda(e, "espace_proj_import: copy");
+    }
+    if (evals) p->evals.assign(evals, evals + K);
+    *out = p;
+    return ESPACE_OK;
+}
+
+void espace_proj_destroy(espace_proj_t p)
+{
+    if (p == nullptr) return;
+    DeviceGuard g(p->device);
+    cudaDeviceSynchronize();
+    if (p->PT) cudaFree(p->PT);
+    if (p->WfT) cudaFree(p->WfT);
+    if (p->Z) cudaFree(p->Z);
+    delete p;
+}
+
+// ---------------------------------------------------------------------------- forward
+
+static int ensure_z(espace_proj_s* p, int64_t N, cudaStream_t st)
+{
+    std::lock_guard<std::mutex> lock(p->mu);
+    if (p->zcap >= N) return ESPACE_OK;
+    CUDA_TRY(cudaStreamSynchronize(st), "forward: sync before scratch growth");
+    if (p->Z) cudaFree(p->Z);
+    p->Z = nullptr;
+    p->zcap = 0;
+    const int64_t cap = std::max<int64_t>(N, 128);
+    cudaError_t e = cudaMalloc(&p->Z, sizeof(uint16_t) * cap * p->Lp);
+    if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "forward: Z scratch of %lld tokens: %s", (long long)cap, cudaGetErrorString(e));
+    p->zcap = cap;
+    return ESPACE_OK;
+}
+
+int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev, void* stream,
+                               int path)
+{
+    if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward: null handle");
+    if (N < 0) return fail(ESPACE_ERR_SHAPE, "espace_linear_forward: N=%lld < 0", (long long)N);
+    if (N == 0) return ESPACE_OK;
+    if (X_dev == nullptr || Y_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward: null pointer");
+    if (!aligned16(X_dev) || !aligned16(Y_dev)) return fail(ESPACE_ERR_ALIGN, "espace_linear_forward: X/Y not 16-byte aligned");
+    if (N > (int64_t(1) << 31) - 256) return fail(ESPACE_ERR_SHAPE, "espace_linear_forward: N=%lld too large", (long long)N);
+    if (path < 0 || path > 2) return fail(ESPACE_ERR_ARG, "espace_linear_forward: unknown path %d", path);
+    const int K = static_cast<int>(p->K), M = static_cast<int>(p->M), Lp = static_cast<int>(p->Lp);
+    const int n = static_cast<int>(N);
+    const bool small_ok = N <= 8 && stream_gemv_supported(n, K) && stream_gemv_supported(n, Lp);
+    if (path == ESPACE_PATH_SMALL_N && !small_ok)
+        return fail(ESPACE_ERR_SHAPE, "espace_linear_forward: N=%lld (K=%d, Lp=%d) beyond the small-N kernels", (long long)N, K, Lp);
+    const bool small = path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok);
+    DeviceGuard g(p->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int rc = ensure_z(p, N, st);
+    if (rc != ESPACE_OK) return rc;
+    cudaEvent_t mid = g_phase_event;
+    g_phase_event = nullptr;
+    if (small) {
+        CUDA_TRY(launch_stream_gemv(p->PT, K, X_dev, K, n, Lp, K, p->Z, Lp, st), "forward: small-N phase 1");
+        if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+        CUDA_TRY(launch_stream_gemv(p->WfT, Lp, p->Z, Lp, n, M, Lp, Y_dev, M, st), "forward: small-N phase 2");
+    } else {
+        CUDA_TRY(launch_gemm_tn(X_dev, K, p->PT, K, n, Lp, K, p->Z, Lp, st), "forward: phase 1");
+        if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+        CUDA_TRY(launch_gemm_tn(p->Z, Lp, p->WfT, Lp, n, M, Lp, Y_dev, M, st), "forward: phase 2");
+    }
+    return ESPACE_OK;
+}
+
+int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev, void* stream)
+{
+    return espace_linear_forward_path(p, X_dev, N, Y_dev, stream, ESPACE_PATH_AUTO);
+}
+
+int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev, int64_t M, void* Y_dev,
+                         void* stream)
+{
+    if (N < 0) return fail(ESPACE_ERR_SHAPE, "espace_dense_forward: N < 0");
+    if (N == 0) return ESPACE_OK;
+    if (X_dev == nullptr || W_dev == nullptr || Y_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_dense_forward: null pointer");
+    if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(Y_dev))
+        return fail(ESPACE_ERR_ALIGN, "espace_dense_forward: pointers must be 16-byte aligned");
+    if (K < 8 || K % 8 != 0 || K > 65536 || M < 8 || M % 8 != 0 || M > (int64_t(1) << 30) || N > (int64_t(1) << 31) - 256)
+        return fail(ESPACE_ERR_SHAPE, "espace_dense_forward: unsupported shape N=%lld K=%lld M=%lld", (long long)N, (long long)K, (long long)M);
+    DeviceInfo* dev = nullptr;
+    int rc = device_info(&dev);
+    if (rc != ESPACE_OK) return rc;
+    CUDA_TRY(launch_gemm_tn(X_dev, K, W_dev, K, static_cast<int>(N), static_cast<int>(M), static_cast<int>(K), Y_dev, M,
+                            static_cast<cudaStream_t>(stream)),
+             "espace_dense_forward: launch");
+    return ESPACE_OK;
+}
+
+int espace_debug_wait_timeout(uint64_t limit_ns, void* stream)
+{
+    if (limit_ns == 0 || limit_ns > 1000000000ull)
+        return fail(ESPACE_ERR_ARG, "espace_debug_wait_timeout: limit must be in (0, 1e9] ns");
+    CUDA_TRY(launch_wait_timeout(limit_ns, static_cast<cudaStream_t>(stream)), "espace_debug_wait_timeout");
+    return ESPACE_OK;
+}
+
+int espace_check(void* stream)
+{
+    DeviceInfo* dev = nullptr;
+    int rc = device_info(&dev);
+    if (rc != ESPACE_OK) return rc;
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "espace_check: stream");
+    int status = 0;
+    CUDA_TRY(cudaMemcpy(&status, dev->status, sizeof(int), cudaMemcpyDeviceToHost), "espace_check: status");
+    if (status != 0) {
+        CUDA_TRY(cudaMemset(dev->status, 0, sizeof(int)), "espace_check: clear");
+        return fail(status, "espace_check: a kernel gave up waiting (device status %d)", status);
+    }
+    return ESPACE_OK;
+}
+
+}  // extern "C"

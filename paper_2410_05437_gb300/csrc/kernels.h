@@ -1,0 +1,47 @@
+// kernels.h -- host-side launchers of the library's CUDA kernels (internal, not the ABI).
+// Every launcher validates nothing: espace_api.cu checks shapes and pointers first.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace espace {
+
+struct DeviceInfo {
+    int device = -1;
+    int num_sms = 0;
+    int* status = nullptr;   // device status word (ESPACE_ERR_TIMEOUT after a failed wait)
+};
+
+// Per-device state, created on first use (the status word is the only allocation).
+int device_info(DeviceInfo** out);
+
+uint64_t wait_limit_ns();
+
+// C[rows][cols] (bf16, leading dimension ldc) = A[rows][kdim] * B[cols][kdim]^T with fp32
+// accumulation on tcgen05 tensor cores; A and B are bf16 with leading dimensions lda, ldb.
+// kdim, lda, ldb and ldc must be multiples of 8 and the pointers 16-byte aligned.
+cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
+                           int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream);
+
+// S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
+cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
+
+// out[n][r] (bf16, leading dimension ldo) = sum_k B[n][k] A[r][k] for n < nt <= 8, with A
+// ([R][kdim], leading dimension lda) streamed once from memory and B ([nt][kdim]) staged
+// in shared memory; fp32 accumulation, warp-level reductions.
+cudaError_t launch_stream_gemv(const void* A, int64_t lda, const void* B, int64_t ldb, int nt,
+                               int R, int kdim, void* out, int64_t ldo, cudaStream_t stream);
+bool stream_gemv_supported(int nt, int kdim);
+
+// Xn[t][k] = bf16(X[t][k] / ||x_t||) (0 for a zero token), fp32 norms.
+cudaError_t launch_normalize_rows(const void* X, int64_t N, int K, void* Xn, cudaStream_t stream);
+
+// One thread waits on an mbarrier that never completes; after limit_ns it records
+// ESPACE_ERR_TIMEOUT in the status word and returns.
+cudaError_t launch_wait_timeout(uint64_t limit_ns, cudaStream_t stream);
+
+// Fills dst[count] with zeros (fp32).
+cudaError_t launch_zero_f32(float* dst, int64_t count, cudaStream_t stream);
+
+}  // namespace espace

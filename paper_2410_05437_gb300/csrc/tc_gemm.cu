@@ -1,0 +1,456 @@
+// tc_gemm.cu -- persistent, warp-specialized tcgen05 GEMM for sm_103a.
+//
+// One CTA per SM loops over output tiles of 128 x BN. Warp 0 (one lane) streams A and B
+// tiles into a STAGES-deep shared-memory ring with TMA (128-byte swizzle); warp 1 (one lane)
+// issues tcgen05.mma (bf16 x bf16 -> fp32) into one of two TMEM accumulators; warps 2-5
+// drain the other accumulator with tcgen05.ld and write the tile, so the epilogue of tile i
+// overlaps the main loop of tile i+1. mbarriers link the roles; every wait is bounded.
+//
+// Two operand layouts share the kernel:
+//   * K-major ("TN"): C[r][c] = sum_k A[r][k] B[c][k] -- the projected layer's two products
+//     Z = X P and Y = Z W' (with P^T and W'^T stored row-major), the fold W'^T = W P and
+//     the dense baseline Y = X W^T;
+//   * M/N-major: S[i][j] += sum_t X[t][i] X[t][j] -- the autocorrelation of Eq. 4, read
+//     straight from token-major X, upper-triangle tiles only, split over tokens with fp32
+//     atomics.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <mutex>
+#include <vector>
+
+#include "../../include/espace.h"
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace espace {
+
+constexpr int BM = 128;                 // UMMA M: rows per tile (= TMEM lanes)
+constexpr int BK = 64;                  // bf16 elements per 128-byte swizzled row
+constexpr int UMMA_K = 16;              // K of one tcgen05.mma.kind::f16
+constexpr int EPI_THREADS = 128;        // 4 epilogue warps, one per TMEM lane quarter
+constexpr int GEMM_THREADS = 64 + EPI_THREADS;
+
+enum { EPI_STORE_BF16 = 0, EPI_ATOMIC_UPPER_F32 = 1 };
+
+struct TcGemmArgs {
+    int rows, cols;        // output extent
+    int kblocks;           // 64-wide blocks along the reduction
+    int tiles_n;           // column tiles (row-major tile grid when tile_list == nullptr)
+    int num_tiles;         // output tiles
+    int ksplit;            // reduction splits per tile (EPI_ATOMIC_UPPER_F32 only)
+    int kb_per_split;
+    const int2* tile_list; // (tile row, tile col) pairs, or nullptr
+    void* out;
+    int64_t ldo;
+    int* status;
+    uint64_t wait_limit_ns;
+};
+
+template <int BN, int STAGES>
+struct TcCfg {
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int TMEM_COLS = 2 * BN;
+    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+    static_assert(STAGE_BYTES % 1024 == 0, "stages must keep 1024-byte alignment");
+    static_assert(TMEM_COLS <= 512, "two accumulators must fit in TMEM");
+};
+
+__device__ __forceinline__ void decode_item(const TcGemmArgs& a, int item, int& tm, int& tn,
+                                            int& kb0, int& kb1)
+{
+    const int tile = item / a.ksplit;
+    const int split = item - tile * a.ksplit;
+    if (a.tile_list != nullptr) {
+        const int2 t = a.tile_list[tile];
+        tm = t.x;
+        tn = t.y;
+    } else {
+        tm = tile / a.tiles_n;
+        tn = tile - tm * a.tiles_n;
+    }
+    kb0 = split * a.kb_per_split;
+    kb1 = min(kb0 + a.kb_per_split, a.kblocks);
+}
+
+template <int BN, int STAGES, bool MN_MAJOR, int EPI>
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap map_a,
+                   const __grid_constant__ CUtensorMap map_b, const TcGemmArgs args)
+{
+    using Cfg = TcCfg<BN, STAGES>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+    uint64_t* empty = full + STAGES;
+    uint64_t* tfull = empty + STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], EPI_THREADS);
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_map(&map_a);
+        tma_prefetch_map(&map_b);
+    }
+    tc_fence_before_sync();
+    __syncthreads();
+    tc_fence_after_sync();
+    const uint32_t tmem_base = *tmem_slot;
+
+    const int num_items = args.num_tiles * args.ksplit;
+    const uint64_t limit = args.wait_limit_ns;
+    volatile int never = 0;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            int armed[STAGES];
+            for (int s = 0; s < STAGES; ++s) armed[s] = -1;
+            bool ok = true;
+            for (int item = blockIdx.x; ok && item < num_items; item += gridDim.x) {
+                int tm, tn, kb0, kb1;
+                decode_item(args, item, tm, tn, kb0, kb1);
+                for (int kb = kb0; kb < kb1; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.status, limit,
+                                   ESPACE_ERR_TIMEOUT)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
+                    uint8_t* sb = sa + Cfg::A_BYTES;
+                    mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
+                    armed[stage] = static_cast<int>(phase);
+                    if (MN_MAJOR) {
+                        // 64 features x 64 tokens per box; box h of a tile at +h*8 KB
+                        tma_load_2d(sa, &map_a, &full[stage], tm * BM, kb * BK);
+                        tma_load_2d(sa + 8192, &map_a, &full[stage], tm * BM + 64, kb * BK);
+#pragma unroll
+                        for (int h = 0; h < BN / 64; ++h)
+                            tma_load_2d(sb + h * 8192, &map_b, &full[stage], tn * BN + h * 64,
+                                        kb * BK);
+                    } else {
+                        tma_load_2d(sa, &map_a, &full[stage], kb * BK, tm * BM);
+                        tma_load_2d(sb, &map_b, &full[stage], kb * BK, tn * BN);
+                    }
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                // let the copies already issued land before the CTA's shared memory goes away
+                for (int s = 0; s < STAGES; ++s)
+                    if (armed[s] >= 0)
+                        mbar_wait(&full[s], static_cast<uint32_t>(armed[s]), &never, args.status,
+                                  limit, ESPACE_ERR_TIMEOUT);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, MN_MAJOR, MN_MAJOR);
+            // K-major: the next 16-element K slice starts 32 bytes further along the
+            // swizzled row. MN-major: 16 tokens further = 16 rows of 128 bytes.
+            constexpr uint32_t k_step = MN_MAJOR ? 2048u : 32u;
+            constexpr uint32_t lbo = MN_MAJOR ? 8192u : 16u;
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int item = blockIdx.x; ok && item < num_items; item += gridDim.x) {
+                int tm, tn, kb0, kb1;
+                decode_item(args, item, tm, tn, kb0, kb1);
+                if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, args.status, limit,
+                               ESPACE_ERR_TIMEOUT))
+                    break;
+                tc_fence_after_sync();
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+                for (int kb = kb0; kb < kb1; ++kb) {
+                    if (!mbar_wait(&full[stage], phase, abort_flag, args.status, limit,
+                                   ESPACE_ERR_TIMEOUT)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after_sync();
+                    const uint32_t a_addr = smem_u32(smem + stage * Cfg::STAGE_BYTES);
+                    const uint32_t b_addr = a_addr + Cfg::A_BYTES;
+#pragma unroll
+                    for (int j = 0; j < BK / UMMA_K; ++j) {
+                        const uint64_t ad = smem_desc_sw128(a_addr + j * k_step, lbo, 1024);
+                        const uint64_t bd = smem_desc_sw128(b_addr + j * k_step, lbo, 1024);
+                        umma_bf16(d_tmem, ad, bd, idesc, (kb > kb0 || j > 0) ? 1u : 0u);
+                    }
+                    umma_commit(&empty[stage]);   // frees the stage once these MMAs finish
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                umma_commit(&tfull[acc]);          // accumulator ready for the epilogue
+                acc ^= 1;
+                if (acc == 0) acc_phase ^= 1u;
+            }
+            // every MMA issued above has finished once this commit arrives
+            umma_commit(drain);
+            mbar_wait(drain, 0, &never, args.status, limit, ESPACE_ERR_TIMEOUT);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (4 warps)
+        const int quarter = warp & 3;            // TMEM lanes this warp may read
+        const int row_in_tile = quarter * 32 + lane;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int item = blockIdx.x; item < num_items; item += gridDim.x) {
+            int tm, tn, kb0, kb1;
+            decode_item(args, item, tm, tn, kb0, kb1);
+            if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, args.status, limit,
+                           ESPACE_ERR_TIMEOUT))
+                break;
+            tc_fence_after_sync();
+            const int row = tm * BM + row_in_tile;
+            const uint32_t t_row =
+                tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(acc * BN);
+#pragma unroll 1
+            for (int c = 0; c < BN; c += 32) {
+                const int col0 = tn * BN + c;
+                if (col0 >= args.cols) break;    // uniform across the warp
+                uint32_t v[32];
+                tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
+                tmem_ld_wait();
+                if (row >= args.rows) continue;
+                if (EPI == EPI_STORE_BF16) {
+                    __nv_bfloat16* out_row =
+                        reinterpret_cast<__nv_bfloat16*>(args.out) + static_cast<int64_t>(row) * args.ldo;
+                    if (col0 + 32 <= args.cols) {
+                        uint4* dst = reinterpret_cast<uint4*>(out_row + col0);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            uint4 q;
+                            q.x = pack_bf16x2(__uint_as_float(v[8 * i + 0]), __uint_as_float(v[8 * i + 1]));
+                            q.y = pack_bf16x2(__uint_as_float(v[8 * i + 2]), __uint_as_float(v[8 * i + 3]));
+                            q.z = pack_bf16x2(__uint_as_float(v[8 * i + 4]), __uint_as_float(v[8 * i + 5]));
+                            q.w = pack_bf16x2(__uint_as_float(v[8 * i + 6]), __uint_as_float(v[8 * i + 7]));
+                            dst[i] = q;
+                        }
+                    } else {
+                        for (int i = 0; i < 32 && col0 + i < args.cols; ++i)
+                            out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
+                    }
+                } else {
+                    float* out_row =
+                        reinterpret_cast<float*>(args.out) + static_cast<int64_t>(row) * args.ldo;
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const int col = col0 + i;
+                        if (col < args.cols && col >= row) atomicAdd(out_row + col, __uint_as_float(v[i]));
+                    }
+                }
+            }
+            tc_fence_before_sync();
+            mbar_arrive(&tempty[acc]);
+            acc ^= 1;
+            if (acc == 0) acc_phase ^= 1u;
+        }
+    }
+
+    tc_fence_before_sync();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after_sync();
+        tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+    }
+}
+
+// =========================================================================== host side
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 2-D bf16 tensor [outer][inner] with a row pitch of `pitch_elems`, 128-byte swizzled boxes
+// of box_inner x box_outer elements, zero fill outside the tensor.
+bool encode_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                uint64_t pitch_elems, uint32_t box_inner, uint32_t box_outer)
+{
+    EncodeTiledFn fn = encode_fn();
+    if (fn == nullptr) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {pitch_elems * 2};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+              box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, int STAGES, bool MN_MAJOR, int EPI>
+cudaError_t launch_kernel(const CUtensorMap& ma, const CUtensorMap& mb, const TcGemmArgs& args,
+                          int grid, cudaStream_t stream)
+{
+    using Cfg = TcCfg<BN, STAGES>;
+    auto kern = tc_gemm_kernel<BN, STAGES, MN_MAJOR, EPI>;
+    static bool attr_set = false;   // per instantiation; benign race (idempotent call)
+    if (!attr_set) {
+        cudaError_t e =
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    kern<<<grid, GEMM_THREADS, Cfg::SMEM_BYTES, stream>>>(ma, mb, args);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
+                           int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream)
+{
+    if (rows <= 0 || cols <= 0) return cudaSuccess;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    const bool wide = cols > 128;
+    const int bn = wide ? 256 : 128;
+    CUtensorMap ma, mb;
+    if (!encode_map(&ma, A, kdim, rows, lda, BK, BM)) return cudaErrorInvalidValue;
+    if (!encode_map(&mb, B, kdim, cols, ldb, BK, bn)) return cudaErrorInvalidValue;
+    TcGemmArgs a{};
+    a.rows = rows;
+    a.cols = cols;
+    a.kblocks = (kdim + BK - 1) / BK;
+    a.tiles_n = (cols + bn - 1) / bn;
+    a.num_tiles = ((rows + BM - 1) / BM) * a.tiles_n;
+    a.ksplit = 1;
+    a.kb_per_split = a.kblocks;
+    a.tile_list = nullptr;
+    a.out = C;
+    a.ldo = ldc;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    const int grid = std::min(a.num_tiles, dev->num_sms);
+    if (wide) return launch_kernel<256, 4, false, EPI_STORE_BF16>(ma, mb, a, grid, stream);
+    return launch_kernel<128, 6, false, EPI_STORE_BF16>(ma, mb, a, grid, stream);
+}
+
+namespace {
+
+struct TileList {
+    int K = -1;
+    int2* dev = nullptr;
+    int count = 0;
+};
+
+// Upper-triangle tile pairs (128-row block, 256-column block) for one K, kept per device.
+int2* syrk_tiles(int K, int* count)
+{
+    static std::mutex mu;
+    static std::vector<std::pair<int, TileList>> cache;   // (device, list)
+    int device = 0;
+    cudaGetDevice(&device);
+    std::lock_guard<std::mutex> lock(mu);
+    for (auto& e : cache)
+        if (e.first == device && e.second.K == K) {
+            *count = e.second.count;
+            return e.second.dev;
+        }
+    std::vector<int2> host;
+    const int tm_n = (K + BM - 1) / BM, tn_n = (K + 255) / 256;
+    for (int tm = 0; tm < tm_n; ++tm)
+        for (int tn = 0; tn < tn_n; ++tn)
+            if (tn * 256 + 255 >= tm * BM) host.push_back(make_int2(tm, tn));
+    int2* dev = nullptr;
+    if (cudaMalloc(&dev, host.size() * sizeof(int2)) != cudaSuccess) return nullptr;
+    if (cudaMemcpy(dev, host.data(), host.size() * sizeof(int2), cudaMemcpyHostToDevice) !=
+        cudaSuccess) {
+        cudaFree(dev);
+        return nullptr;
+    }
+    TileList t;
+    t.K = K;
+    t.dev = dev;
+    t.count = static_cast<int>(host.size());
+    cache.emplace_back(device, t);
+    *count = t.count;
+    return dev;
+}
+
+}  // namespace
+
+cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream)
+{
+    if (N <= 0) return cudaSuccess;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    int count = 0;
+    const int2* tiles = syrk_tiles(K, &count);
+    if (tiles == nullptr) return cudaErrorMemoryAllocation;
+    CUtensorMap mx;
+    if (!encode_map(&mx, X, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
+    TcGemmArgs a{};
+    a.rows = K;
+    a.cols = K;
+    a.kblocks = static_cast<int>((N + BK - 1) / BK);
+    a.tiles_n = 0;
+    a.num_tiles = count;
+    // split the tokens so that there are about two work items per SM, at least 16 blocks
+    // (1024 tokens) per split
+    int want_splits = std::max(1, (2 * dev->num_sms + count - 1) / count);
+    int kbps = std::max(16, (a.kblocks + want_splits - 1) / want_splits);
+    kbps = std::min(kbps, a.kblocks);
+    a.kb_per_split = kbps;
+    a.ksplit = (a.kblocks + kbps - 1) / kbps;
+    a.tile_list = tiles;
+    a.out = S;
+    a.ldo = K;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    const int grid = std::min(a.num_tiles * a.ksplit, dev->num_sms);
+    return launch_kernel<256, 4, true, EPI_ATOMIC_UPPER_F32>(mx, mx, a, grid, stream);
+}
+
+}  // namespace espace

@@ -129,6 +129,27 @@ class ActivationModel:
         """``n`` tokens as a bf16 ``[n, K]`` CPU tensor."""
         return to_bf16(self.sample_f32(n, stream, chunk))
 
+    def sample_device(self, n: int, stream: str = "eval_tokens", chunk: int = 0,
+                      device: str = "cuda") -> torch.Tensor:
+        """Same recipe drawn on the GPU with torch's Philox generator (a different random
+        stream from ``sample``): for benchmark inputs too large to draw on the host. Not
+        used where an oracle value is compared."""
+        gen = torch.Generator(device=device)
+        gen.manual_seed((int(self.seed) * 1000003 + _STREAMS[stream] * 7919 + int(chunk)) % (1 << 63))
+        g = torch.randn((n, self.K), generator=gen, device=device, dtype=torch.float32)
+        y = g * torch.as_tensor(self.spectrum, dtype=torch.float32, device=device)
+        if self._rot == "haar":
+            if getattr(self, "_QT_dev", None) is None or self._QT_dev.device != y.device:
+                self._QT_dev = torch.as_tensor(self._QT32, device=device)
+            y = y @ self._QT_dev
+        else:
+            for v in self._reflectors:
+                vt = torch.as_tensor(v, device=device)
+                y = y - 2.0 * (y @ vt)[:, None] * vt[None, :]
+            y = y[:, torch.as_tensor(self._perm, device=device)] * torch.as_tensor(self._signs, device=device)
+        y = y * torch.as_tensor(self.channel_scale, dtype=torch.float32, device=device)
+        return y.to(torch.bfloat16)
+
     def sample_gated(self, n: int, chunk: int = 0) -> torch.Tensor:
         """Down-projection input ``silu(a) * b`` (fp32, then bf16) with independent a, b."""
         a = self.sample_f32(n, "gate_a", chunk)
@@ -141,6 +162,15 @@ def weights(M: int, K: int, seed: int = BASE_SEED, chunk: int = 0) -> torch.Tens
     """``W`` as bf16 ``[M, K]`` (PyTorch Linear layout), iid N(0, 1/K)."""
     w = generator(seed, "weights", chunk).standard_normal((M, K), dtype=np.float32)
     return to_bf16(w * np.float32(1.0 / math.sqrt(K)))
+
+
+def weights_device(M: int, K: int, seed: int = BASE_SEED, chunk: int = 0,
+                   device: str = "cuda") -> torch.Tensor:
+    """``W`` drawn on the GPU (benchmark inputs only; see ``ActivationModel.sample_device``)."""
+    gen = torch.Generator(device=device)
+    gen.manual_seed((int(seed) * 1000003 + _STREAMS["weights"] * 7919 + int(chunk)) % (1 << 63))
+    w = torch.randn((M, K), generator=gen, device=device, dtype=torch.float32)
+    return (w * (1.0 / math.sqrt(K))).to(torch.bfloat16)
 
 
 def random_projection(K: int, L: int, seed: int = BASE_SEED) -> np.ndarray:
