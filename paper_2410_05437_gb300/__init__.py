@@ -5,7 +5,7 @@ Argument marshalling only: every function below forwards to the C ABI of the sam
 tensors into device pointers, streams into ``cudaStream_t`` handles and non-zero return
 codes into :class:`EspaceError`. All arithmetic runs in the library's CUDA kernels (and its
 host eigen-solver); there is no Python or CPU fallback, and importing this package fails if
-the library has not been built (``python -m paper_2410_05437_gb300.build``).
+the library has not been built (``python paper_2410_05437_gb300/build.py``).
 
 Layouts follow the ABI: ``X`` is ``[N, K]``, ``W`` is ``[M, K]`` (``nn.Linear``), ``Y`` is
 ``[N, M]``, all bf16 and contiguous on the GPU.
@@ -48,7 +48,7 @@ class EspaceError(RuntimeError):
 if not os.path.exists(LIBRARY_PATH):
     raise ImportError(
         f"{LIBRARY_PATH} is missing: build the CUDA library first "
-        "(python -m paper_2410_05437_gb300.build)")
+        "(python paper_2410_05437_gb300/build.py, or __graft_entry__.build())")
 
 lib = ctypes.CDLL(LIBRARY_PATH)
 
