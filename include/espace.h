@@ -162,6 +162,28 @@ int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y
 int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev,
                                void* stream, int path);
 
+/* Capacity, in bf16 values, of the fixed scratch used by espace_linear_forward_noalloc:
+ * 16 MiB, enough for N * Lp <= 8,388,608 (e.g. 4096 tokens at L = 2048). */
+#define ESPACE_NOALLOC_Z_ELEMS 8388608
+
+/* Async. Same result as espace_linear_forward (automatic path) for callers that cannot
+ * allocate device memory during the call -- for example code that runs inside a memory
+ * budget or pool owned by someone else, or a server that reserved all device memory at
+ * start-up. Instead of the handle's growable Z scratch it uses one fixed array of
+ * ESPACE_NOALLOC_Z_ELEMS bf16 values that is part of the library image on every device
+ * that loads the library (held until the process exits); the call itself allocates
+ * nothing. The paper has no counterpart: it is an interface convenience of this library.
+ *   - N * Lp (Lp = L rounded up to a multiple of 64) above ESPACE_NOALLOC_Z_ELEMS is
+ *     rejected with ESPACE_ERR_SHAPE before anything is launched.
+ *   - The handle's device must be current (ESPACE_ERR_STATE otherwise).
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - All calls on a device share the array and it keeps the last call's contents (each
+ *     call overwrites the part it reads); calls whose kernels overlap on the GPU, e.g. on
+ *     two unordered streams, race on it. */
+int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev,
+                                  void* stream);
+
 /* Async. The uncompressed layer of Eq. 1, Y = W^T X, as Y_dev[N][M] = X_dev[N][K] W_dev^T
  * with W_dev in [M][K] layout, on the same tcgen05 kernel with fp32 accumulation and bf16
  * output: the baseline the projected layer is measured against. */

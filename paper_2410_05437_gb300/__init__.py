@@ -27,7 +27,8 @@ __all__ = [
     "espace_build_projection", "espace_proj_from_host", "espace_proj_shape",
     "espace_proj_eigenvalues", "espace_proj_read_P", "espace_proj_read_Wfold",
     "espace_proj_export", "espace_proj_import", "espace_proj_destroy",
-    "espace_linear_forward", "espace_linear_forward_path", "espace_dense_forward",
+    "espace_linear_forward", "espace_linear_forward_path", "espace_linear_forward_noalloc",
+    "espace_dense_forward",
     "espace_check", "espace_debug_wait_timeout", "espace_set_wait_limit_ns", "espace_set_phase_event",
     "espace_host_eigh",
     "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "EXPORTED_SYMBOLS",
@@ -82,6 +83,7 @@ _SIGNATURES = {
     "espace_proj_destroy": (None, [_vp]),
     "espace_linear_forward": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_linear_forward_path": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp, ctypes.c_int]),
+    "espace_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_dense_forward": (ctypes.c_int, [_vp, _i64, _i64, _vp, _i64, _vp, _vp]),
     "espace_check": (ctypes.c_int, [_vp]),
     "espace_debug_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _vp]),
@@ -289,6 +291,13 @@ def espace_linear_forward_path(p: int, X, Y, path: int, N: int | None = None, st
     N = X.shape[0] if N is None else N
     _check(lib.espace_linear_forward_path(p, _dev_ptr(X), int(N), _dev_ptr(Y), _stream(stream),
                                           int(path)))
+
+
+def espace_linear_forward_noalloc(p: int, X, Y, N: int | None = None, stream=None) -> None:
+    """Forward that allocates nothing during the call (fixed library-owned Z scratch); for
+    callers that may not allocate device memory at that point. See include/espace.h."""
+    N = X.shape[0] if N is None else N
+    _check(lib.espace_linear_forward_noalloc(p, _dev_ptr(X), int(N), _dev_ptr(Y), _stream(stream)))
 
 
 def espace_dense_forward(X, W, Y, stream=None) -> None:

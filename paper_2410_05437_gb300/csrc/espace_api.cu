@@ -643,3 +643,31 @@ int espace_check(void* stream)
 }
 
 }  // extern "C"
+
+// ============================================================================ internal views
+
+namespace espace {
+
+struct ProjView {
+    int64_t K, M, L, Lp;
+    int device;
+    const void* PT;
+    const void* WfT;
+};
+
+int proj_view(espace_proj_t p, ProjView* out)
+{
+    if (p == nullptr || out == nullptr) return fail(ESPACE_ERR_ARG, "proj_view: null pointer");
+    out->K = p->K;
+    out->M = p->M;
+    out->L = p->L;
+    out->Lp = p->Lp;
+    out->device = p->device;
+    out->PT = p->PT;
+    out->WfT = p->WfT;
+    return ESPACE_OK;
+}
+
+void set_last_error(const char* msg) { g_last_error = msg; }
+
+}  // namespace espace
