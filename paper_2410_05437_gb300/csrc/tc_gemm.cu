@@ -16,6 +16,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <stdlib.h>
+
 #include <algorithm>
 #include <mutex>
 #include <vector>
@@ -58,6 +60,14 @@ struct TcCfg {
     static_assert(STAGE_BYTES % 1024 == 0, "stages must keep 1024-byte alignment");
     static_assert(TMEM_COLS <= 512, "two accumulators must fit in TMEM");
 };
+
+// After a producer gave up, copies it already issued may still be landing in shared
+// memory: wait 200 us (far longer than any copy takes) before the CTA can exit.
+__device__ __forceinline__ void settle_copies()
+{
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 200000ull) __nanosleep(1000);
+}
 
 __device__ __forceinline__ void decode_item(const TcGemmArgs& a, int item, int& tm, int& tn,
                                             int& kb0, int& kb1)
@@ -121,15 +131,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 
     const int num_items = args.num_tiles * args.ksplit;
     const uint64_t limit = args.wait_limit_ns;
-    volatile int never = 0;
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
-            int armed[STAGES];
-            for (int s = 0; s < STAGES; ++s) armed[s] = -1;
             bool ok = true;
             for (int item = blockIdx.x; ok && item < num_items; item += gridDim.x) {
                 int tm, tn, kb0, kb1;
@@ -143,7 +150,6 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                     uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
                     uint8_t* sb = sa + Cfg::A_BYTES;
                     mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
-                    armed[stage] = static_cast<int>(phase);
                     if (MN_MAJOR) {
                         // 64 features x 64 tokens per box; box h of a tile at +h*8 KB
                         tma_load_2d(sa, &map_a, &full[stage], tm * BM, kb * BK);
@@ -162,13 +168,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                     }
                 }
             }
-            if (!ok) {
-                // let the copies already issued land before the CTA's shared memory goes away
-                for (int s = 0; s < STAGES; ++s)
-                    if (armed[s] >= 0)
-                        mbar_wait(&full[s], static_cast<uint32_t>(armed[s]), &never, args.status,
-                                  limit, ESPACE_ERR_TIMEOUT);
-            }
+            if (!ok) settle_copies();
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -219,6 +219,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             }
             // every MMA issued above has finished once this commit arrives
             umma_commit(drain);
+            volatile int never = 0;
             mbar_wait(drain, 0, &never, args.status, limit, ESPACE_ERR_TIMEOUT);
         }
     } else {
@@ -260,8 +261,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                             dst[i] = q;
                         }
                     } else {
-                        for (int i = 0; i < 32 && col0 + i < args.cols; ++i)
-                            out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (col0 + i < args.cols)
+                                out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
                     }
                 } else {
                     float* out_row =
@@ -280,11 +283,223 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
     }
 
+    __syncwarp();
     tc_fence_before_sync();
     __syncthreads();
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+    }
+}
+
+// =========================================================================== CTA-pair kernel
+//
+// Same pipeline on a pair of CTAs (a cluster of two on neighbouring SMs) computing
+// 256 x 256 output tiles with tcgen05.mma.cta_group::2: each CTA stages 128 rows of A and
+// 128 rows (half) of B per k-block, so each SM moves 32 KB instead of 48 KB of operands per
+// 64-deep k-block for twice the tile. The leader CTA (rank 0) issues the MMAs for both; the
+// two producers count their copies on the leader's "full" barrier; the leader's commits
+// arrive on both CTAs' "empty" and "accumulator full" barriers; each CTA drains its own
+// TMEM half (rows rank*128 .. +128 of the tile) and releases the accumulator on the
+// leader's barrier.
+constexpr int PAIR_BM = 256;        // tile rows per pair (128 per CTA)
+constexpr int PAIR_BN = 256;        // tile columns per pair (B rows: 128 per CTA)
+constexpr int PAIR_STAGES = 6;
+constexpr int PAIR_A_BYTES = 128 * BK * 2;
+constexpr int PAIR_B_BYTES = 128 * BK * 2;
+constexpr int PAIR_STAGE_BYTES = PAIR_A_BYTES + PAIR_B_BYTES;
+constexpr int PAIR_ACCS = 2;        // TMEM accumulators per CTA (1 or 2)
+constexpr int PAIR_TMEM_COLS = PAIR_ACCS * PAIR_BN;
+constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 256;
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
+    tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a,
+                        const __grid_constant__ CUtensorMap map_b, const TcGemmArgs args)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + PAIR_STAGES * PAIR_STAGE_BYTES);
+    uint64_t* empty = full + PAIR_STAGES;
+    uint64_t* tfull = empty + PAIR_STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const bool leader = rank == 0;
+    const int pair = static_cast<int>(blockIdx.x >> 1);
+    const int npairs = static_cast<int>(gridDim.x >> 1);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < PAIR_STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], 2 * EPI_THREADS);   // both CTAs' epilogue threads
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) tmem_alloc_pair(tmem_slot, PAIR_TMEM_COLS);
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_map(&map_a);
+        tma_prefetch_map(&map_b);
+    }
+    tc_fence_before_sync();
+    cluster_sync();   // barriers of both CTAs initialised before any remote arrive or copy
+    tc_fence_after_sync();
+    const uint32_t tmem_base = *tmem_slot;
+    // The pair's MMAs write the accumulator at the leader's TMEM address in both CTAs, so
+    // both allocations must have returned the same address; if not, do no work and report.
+    const uint32_t peer_base = ld_shared_cluster_u32(mapa_shared(smem_u32(tmem_slot), rank ^ 1u));
+    const bool tmem_agree = peer_base == tmem_base;
+    if (!tmem_agree && threadIdx.x == 0) atomicExch(args.status, ESPACE_ERR_STATE);
+
+    const int num_items = tmem_agree ? args.num_tiles : 0;
+    const uint64_t limit = args.wait_limit_ns;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer (both CTAs)
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            for (int item = pair; ok && item < num_items; item += npairs) {
+                const int tm = item / args.tiles_n, tn = item - (item / args.tiles_n) * args.tiles_n;
+                const int row_a = tm * PAIR_BM + static_cast<int>(rank) * 128;
+                const int row_b = tn * PAIR_BN + static_cast<int>(rank) * 128;
+                for (int kb = 0; kb < args.kblocks; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.status, limit,
+                                   ESPACE_ERR_TIMEOUT)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* sa = smem + stage * PAIR_STAGE_BYTES;
+                    uint8_t* sb = sa + PAIR_A_BYTES;
+                    if (leader) mbar_arrive_expect_tx(&full[stage], 2 * PAIR_STAGE_BYTES);
+                    const uint32_t bar = mapa_shared(smem_u32(&full[stage]), 0);
+                    tma_load_2d_pair(sa, &map_a, bar, kb * BK, row_a);
+                    tma_load_2d_pair(sb, &map_b, bar, kb * BK, row_b);
+                    if (++stage == PAIR_STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) settle_copies();
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer (leader)
+        if (lane == 0 && leader) {
+            constexpr uint32_t idesc = idesc_bf16_f32(PAIR_BM, PAIR_BN, false, false);
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int item = pair; ok && item < num_items; item += npairs) {
+                if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, args.status, limit,
+                               ESPACE_ERR_TIMEOUT))
+                    break;
+                tc_fence_after_sync();
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * PAIR_BN);
+                for (int kb = 0; kb < args.kblocks; ++kb) {
+                    if (!mbar_wait(&full[stage], phase, abort_flag, args.status, limit,
+                                   ESPACE_ERR_TIMEOUT)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after_sync();
+                    const uint32_t a_addr = smem_u32(smem + stage * PAIR_STAGE_BYTES);
+                    const uint32_t b_addr = a_addr + PAIR_A_BYTES;
+#pragma unroll
+                    for (int j = 0; j < BK / UMMA_K; ++j) {
+                        const uint64_t ad = smem_desc_sw128(a_addr + j * 32, 16, 1024);
+                        const uint64_t bd = smem_desc_sw128(b_addr + j * 32, 16, 1024);
+                        umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > 0 || j > 0) ? 1u : 0u);
+                    }
+                    umma_commit_pair(&empty[stage], 0x3);   // frees the stage in both CTAs
+                    if (++stage == PAIR_STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                umma_commit_pair(&tfull[acc], 0x3);          // both halves ready to drain
+                if (++acc == PAIR_ACCS) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+            }
+            umma_commit_pair(drain, 0x1);
+            volatile int never = 0;
+            mbar_wait(drain, 0, &never, args.status, limit, ESPACE_ERR_TIMEOUT);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (both CTAs)
+        const int quarter = warp & 3;
+        const int row_in_tile = static_cast<int>(rank) * 128 + quarter * 32 + lane;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int item = pair; item < num_items; item += npairs) {
+            const int tm = item / args.tiles_n, tn = item - (item / args.tiles_n) * args.tiles_n;
+            if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, args.status, limit,
+                           ESPACE_ERR_TIMEOUT))
+                break;
+            tc_fence_after_sync();
+            const int row = tm * PAIR_BM + row_in_tile;
+            const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                   static_cast<uint32_t>(acc * PAIR_BN);
+            __nv_bfloat16* out_row =
+                reinterpret_cast<__nv_bfloat16*>(args.out) + static_cast<int64_t>(row) * args.ldo;
+#pragma unroll 1
+            for (int c = 0; c < PAIR_BN; c += 32) {
+                const int col0 = tn * PAIR_BN + c;
+                if (col0 >= args.cols) break;        // uniform across the warp
+                uint32_t v[32];
+                tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
+                tmem_ld_wait();
+                if (row >= args.rows) continue;
+                if (col0 + 32 <= args.cols) {
+                    uint4* dst = reinterpret_cast<uint4*>(out_row + col0);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        uint4 q;
+                        q.x = pack_bf16x2(__uint_as_float(v[8 * i + 0]), __uint_as_float(v[8 * i + 1]));
+                        q.y = pack_bf16x2(__uint_as_float(v[8 * i + 2]), __uint_as_float(v[8 * i + 3]));
+                        q.z = pack_bf16x2(__uint_as_float(v[8 * i + 4]), __uint_as_float(v[8 * i + 5]));
+                        q.w = pack_bf16x2(__uint_as_float(v[8 * i + 6]), __uint_as_float(v[8 * i + 7]));
+                        dst[i] = q;
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        if (col0 + i < args.cols)
+                            out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
+                }
+            }
+            tc_fence_before_sync();
+            mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[acc]), 0));
+            if (++acc == PAIR_ACCS) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+    }
+
+    __syncwarp();
+    tc_fence_before_sync();
+    cluster_sync();   // no CTA leaves while its peer may still touch its barriers or TMEM
+    if (warp == 1) {
+        tc_fence_after_sync();
+        tmem_dealloc_pair(tmem_base, PAIR_TMEM_COLS);
     }
 }
 
@@ -346,6 +561,49 @@ cudaError_t launch_kernel(const CUtensorMap& ma, const CUtensorMap& mb, const Tc
     return cudaGetLastError();
 }
 
+// 256 x 256 tiles on CTA pairs; grid = 2 x min(tiles, SMs / 2).
+cudaError_t launch_gemm_tn_pair(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
+                                int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream,
+                                const DeviceInfo* dev)
+{
+    CUtensorMap ma, mb;
+    if (!encode_map(&ma, A, kdim, rows, lda, BK, 128)) return cudaErrorInvalidValue;
+    if (!encode_map(&mb, B, kdim, cols, ldb, BK, 128)) return cudaErrorInvalidValue;
+    TcGemmArgs a{};
+    a.rows = rows;
+    a.cols = cols;
+    a.kblocks = (kdim + BK - 1) / BK;
+    a.tiles_n = (cols + PAIR_BN - 1) / PAIR_BN;
+    a.num_tiles = ((rows + PAIR_BM - 1) / PAIR_BM) * a.tiles_n;
+    a.ksplit = 1;
+    a.kb_per_split = a.kblocks;
+    a.tile_list = nullptr;
+    a.out = C;
+    a.ldo = ldc;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    const int pairs = std::min(a.num_tiles, dev->num_sms / 2);
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, PAIR_SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    tc_gemm_pair_kernel<<<2 * pairs, GEMM_THREADS, PAIR_SMEM_BYTES, stream>>>(ma, mb, a);
+    return cudaGetLastError();
+}
+
+// The CTA-pair kernel is used unless ESPACE_DISABLE_PAIR_GEMM=1 is set in the environment.
+bool pair_kernel_enabled()
+{
+    static const bool enabled = [] {
+        const char* v = getenv("ESPACE_DISABLE_PAIR_GEMM");
+        return !(v != nullptr && v[0] == '1');
+    }();
+    return enabled;
+}
+
 }  // namespace
 
 cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
@@ -354,6 +612,8 @@ cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ld
     if (rows <= 0 || cols <= 0) return cudaSuccess;
     DeviceInfo* dev = nullptr;
     if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    if (rows > 128 && cols > 128 && dev->num_sms >= 2 && pair_kernel_enabled())
+        return launch_gemm_tn_pair(A, lda, B, ldb, rows, cols, kdim, C, ldc, stream, dev);
     const bool wide = cols > 128;
     const int bn = wide ? 256 : 128;
     CUtensorMap ma, mb;
