@@ -363,23 +363,55 @@ def side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, espa
                                 "frac_tensor_peak": cflops / cal_ms / 1e9 / peak_tc}
     esp.espace_calib_destroy(h)
     del Xc
-    # decode-shaped forward at N = 1 (small-N streaming kernels)
-    x1 = [s["X"][:1].contiguous() for s in sets]
-    y1 = torch.empty((1, M), dtype=torch.bfloat16, device="cuda")
-    for i in range(3):
-        esp.espace_linear_forward(sets[i % SETS]["p"], x1[i % SETS], y1)
+    # decode-shaped forward, N = 1 .. 512 tokens: ESPACE and dense, each replayed from a
+    # CUDA graph of 20 calls so that host launch overhead is not in the GPU time
+    Lp = (L + 63) // 64 * 64
+    sweep = {}
+    for n_tok in synth.DECODE_TOKENS:
+        xs = [s["X"][:n_tok].contiguous() for s in sets]
+        ys = [torch.empty((n_tok, M), dtype=torch.bfloat16, device="cuda") for _ in sets]
+
+        def espace_call(i, xs=xs, ys=ys):
+            esp.espace_linear_forward(sets[i % SETS]["p"], xs[i % SETS], ys[i % SETS])
+
+        def dense_call(i, xs=xs, ys=ys):
+            esp.espace_dense_forward(xs[i % SETS], sets[i % SETS]["W"], ys[i % SETS])
+
+        e_us = graph_time_us(espace_call)
+        d_us = graph_time_us(dense_call)
+        ebytes = 2.0 * (K * Lp + Lp * M + n_tok * (K + M))
+        dbytes = 2.0 * (K * M + n_tok * (K + M))
+        sweep[str(n_tok)] = {
+            "espace_us": e_us, "dense_us": d_us, "speedup": d_us / e_us,
+            "espace_gbs": ebytes / e_us / 1e3, "espace_frac_hbm": ebytes / e_us / 1e3 / peak_hbm,
+            "espace_tflops": 2.0 * n_tok * (K * L + L * M) / e_us / 1e6,
+            "dense_gbs": dbytes / d_us / 1e3, "path": "decode kernel" if n_tok <= 8 else "tcgen05"}
+    rows["decode_sweep_llama2_qkv"] = sweep
+    return rows
+
+
+def graph_time_us(call, per_graph=20, replays=10):
+    """Mean GPU time of one call, from CUDA-graph replays (inputs rotate inside the graph)."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for i in range(3):
+            call(i)
+    torch.cuda.current_stream().wait_stream(side)
     torch.cuda.synchronize()
-    drep = 200
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for i in range(per_graph):
+            call(i)
+    g.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record()
-    for i in range(drep):
-        esp.espace_linear_forward(sets[i % SETS]["p"], x1[i % SETS], y1)
+    for _ in range(replays):
+        g.replay()
     b.record()
     torch.cuda.synchronize()
-    d_ms = a.elapsed_time(b) / drep
-    Lp = (L + 63) // 64 * 64
-    dbytes = 2.0 * (K * Lp + Lp * M + K + M)
-    rows["decode_n1"] = {"us": d_ms * 1e3, "gbs": dbytes / d_ms / 1e6, "frac_hbm": dbytes / d_ms / 1e6 / peak_hbm}
-    return rows
+    return a.elapsed_time(b) * 1e3 / (per_graph * replays)
 
 
 def main():

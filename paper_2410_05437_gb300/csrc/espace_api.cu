@@ -169,6 +169,7 @@ struct espace_proj_s {
     std::vector<double> evals;     // K eigenvalues, decreasing (if calibrated)
     uint16_t* Z = nullptr;         // [zcap][Lp] bf16 scratch for the rank-L intermediate
     int64_t zcap = 0;
+    unsigned int* bar = nullptr;   // grid barrier of the decode kernel (2 words, zeroed)
     std::mutex mu;                 // guards Z growth
 };
 
@@ -365,8 +366,12 @@ static int proj_create(int64_t K, int64_t M, int64_t L, espace_proj_s** out)
     p->device = dev->device;
     cudaError_t e = cudaMalloc(&p->PT, sizeof(uint16_t) * p->Lp * K);
     if (e == cudaSuccess) e = cudaMalloc(&p->WfT, sizeof(uint16_t) * M * p->Lp);
+    if (e == cudaSuccess) e = cudaMalloc(&p->bar, 64);
+    if (e == cudaSuccess) e = cudaMemset(p->bar, 0, 64);
     if (e != cudaSuccess) {
         if (p->PT) cudaFree(p->PT);
+        if (p->WfT) cudaFree(p->WfT);
+        if (p->bar) cudaFree(p->bar);
         delete p;
         return fail(ESPACE_ERR_NOMEM, "projection: cudaMalloc: %s", cudaGetErrorString(e));
     }
@@ -541,6 +546,7 @@ void espace_proj_destroy(espace_proj_t p)
     if (p->PT) cudaFree(p->PT);
     if (p->WfT) cudaFree(p->WfT);
     if (p->Z) cudaFree(p->Z);
+    if (p->bar) cudaFree(p->bar);
     delete p;
 }
 
@@ -573,7 +579,13 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
     if (path < 0 || path > 2) return fail(ESPACE_ERR_ARG, "espace_linear_forward: unknown path %d", path);
     const int K = static_cast<int>(p->K), M = static_cast<int>(p->M), Lp = static_cast<int>(p->Lp);
     const int n = static_cast<int>(N);
-    const bool small_ok = N <= 8 && stream_gemv_supported(n, K) && stream_gemv_supported(n, Lp);
+    DeviceInfo* dev = nullptr;
+    {
+        DeviceGuard g0(p->device);
+        int rc0 = device_info(&dev);
+        if (rc0 != ESPACE_OK) return rc0;
+    }
+    const bool small_ok = N <= DECODE_MAX_TOKENS && decode_supported(n, K, Lp, M, dev->num_sms);
     if (path == ESPACE_PATH_SMALL_N && !small_ok)
         return fail(ESPACE_ERR_SHAPE, "espace_linear_forward: N=%lld (K=%d, Lp=%d) beyond the small-N kernels", (long long)N, K, Lp);
     const bool small = path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok);
@@ -584,9 +596,10 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
     cudaEvent_t mid = g_phase_event;
     g_phase_event = nullptr;
     if (small) {
-        CUDA_TRY(launch_stream_gemv(p->PT, K, X_dev, K, n, Lp, K, p->Z, Lp, st), "forward: small-N phase 1");
+        // one launch holds both products; the phase event marks its end
+        CUDA_TRY(launch_decode_forward(p->PT, p->WfT, X_dev, p->Z, Y_dev, K, Lp, M, n, p->bar, st),
+                 "forward: decode kernel");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
-        CUDA_TRY(launch_stream_gemv(p->WfT, Lp, p->Z, Lp, n, M, Lp, Y_dev, M, st), "forward: small-N phase 2");
     } else {
         CUDA_TRY(launch_gemm_tn(X_dev, K, p->PT, K, n, Lp, K, p->Z, Lp, st), "forward: phase 1");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
@@ -613,6 +626,13 @@ int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_
     DeviceInfo* dev = nullptr;
     int rc = device_info(&dev);
     if (rc != ESPACE_OK) return rc;
+    // few tokens: stream W once through the decode kernel; otherwise the tcgen05 GEMM
+    if (N <= DECODE_MAX_TOKENS && decode_supported(static_cast<int>(N), static_cast<int>(K), 8, static_cast<int>(M), dev->num_sms)) {
+        CUDA_TRY(launch_decode_dense(W_dev, X_dev, Y_dev, static_cast<int>(K), static_cast<int>(M), static_cast<int>(N),
+                                     static_cast<cudaStream_t>(stream)),
+                 "espace_dense_forward: decode launch");
+        return ESPACE_OK;
+    }
     CUDA_TRY(launch_gemm_tn(X_dev, K, W_dev, K, static_cast<int>(N), static_cast<int>(M), static_cast<int>(K), Y_dev, M,
                             static_cast<cudaStream_t>(stream)),
              "espace_dense_forward: launch");
@@ -653,6 +673,7 @@ struct ProjView {
     int device;
     const void* PT;
     const void* WfT;
+    unsigned int* bar;
 };
 
 int proj_view(espace_proj_t p, ProjView* out)
@@ -665,6 +686,7 @@ int proj_view(espace_proj_t p, ProjView* out)
     out->device = p->device;
     out->PT = p->PT;
     out->WfT = p->WfT;
+    out->bar = p->bar;
     return ESPACE_OK;
 }
 

@@ -27,12 +27,20 @@ cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ld
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
 
-// out[n][r] (bf16, leading dimension ldo) = sum_k B[n][k] A[r][k] for n < nt <= 8, with A
-// ([R][kdim], leading dimension lda) streamed once from memory and B ([nt][kdim]) staged
-// in shared memory; fp32 accumulation, warp-level reductions.
-cudaError_t launch_stream_gemv(const void* A, int64_t lda, const void* B, int64_t ldb, int nt,
-                               int R, int kdim, void* out, int64_t ldo, cudaStream_t stream);
-bool stream_gemv_supported(int nt, int kdim);
+// Token counts served by the decode kernels.
+constexpr int DECODE_MAX_TOKENS = 32;
+
+// Decode-shaped forward (nt <= DECODE_MAX_TOKENS) in one cooperative launch: Z[nt][Lp] = X P
+// from P^T [Lp][K], a grid barrier, then Y[nt][M] = Z W' from W'^T [M][Lp]; each matrix
+// streamed from HBM once. grid_bar: two zeroed unsigned ints owned by the caller (one launch
+// at a time may use them).
+cudaError_t launch_decode_forward(const void* PT, const void* WfT, const void* X, void* Z, void* Y,
+                                  int K, int Lp, int M, int nt, unsigned int* grid_bar,
+                                  cudaStream_t stream);
+// Dense decode product Y[nt][M] = X W^T with W [M][K] streamed once (same kernel, one phase).
+cudaError_t launch_decode_dense(const void* W, const void* X, void* Y, int K, int M, int nt,
+                                cudaStream_t stream);
+bool decode_supported(int nt, int K, int Lp, int M, int num_sms);
 
 // Xn[t][k] = bf16(X[t][k] / ||x_t||) (0 for a zero token), fp32 norms.
 cudaError_t launch_normalize_rows(const void* X, int64_t N, int K, void* Xn, cudaStream_t stream);

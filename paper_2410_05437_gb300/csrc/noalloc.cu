@@ -33,6 +33,7 @@ struct ProjView {
     int device;
     const void* PT;
     const void* WfT;
+    unsigned int* bar;
 };
 int proj_view(espace_proj_t p, ProjView* out);
 void set_last_error(const char* msg);   // espace_last_error() text of the calling thread
@@ -111,11 +112,13 @@ extern "C" int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev,
     const int K = static_cast<int>(v.K), M = static_cast<int>(v.M), Lp = static_cast<int>(v.Lp);
     const int n = static_cast<int>(N);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const bool small = N <= 8 && stream_gemv_supported(n, K) && stream_gemv_supported(n, Lp);
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, v.device) != cudaSuccess)
+        return fail(ESPACE_ERR_CUDA, "espace_linear_forward_noalloc: device query failed");
+    const bool small = N <= DECODE_MAX_TOKENS && decode_supported(n, K, Lp, M, sms);
     cudaError_t e;
     if (small) {
-        e = launch_stream_gemv(v.PT, K, X_dev, K, n, Lp, K, Z, Lp, st);
-        if (e == cudaSuccess) e = launch_stream_gemv(v.WfT, Lp, Z, Lp, n, M, Lp, Y_dev, M, st);
+        e = launch_decode_forward(v.PT, v.WfT, X_dev, Z, Y_dev, K, Lp, M, n, v.bar, st);
     } else {
         e = launch_gemm_tn(X_dev, K, v.PT, K, n, Lp, K, Z, Lp, st);
         if (e == cudaSuccess) e = launch_gemm_tn(Z, Lp, v.WfT, Lp, n, M, Lp, Y_dev, M, st);

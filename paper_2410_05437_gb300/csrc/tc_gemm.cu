@@ -550,12 +550,16 @@ cudaError_t launch_kernel(const CUtensorMap& ma, const CUtensorMap& mb, const Tc
 {
     using Cfg = TcCfg<BN, STAGES>;
     auto kern = tc_gemm_kernel<BN, STAGES, MN_MAJOR, EPI>;
-    static bool attr_set = false;   // per instantiation; benign race (idempotent call)
-    if (!attr_set) {
+    // per instantiation and device; a race only repeats the idempotent call
+    static bool attr_set[64] = {};
+    int device = 0;
+    cudaGetDevice(&device);
+    if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
+    if (!attr_set[device]) {
         cudaError_t e =
             cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM_BYTES);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr_set[device] = true;
     }
     kern<<<grid, GEMM_THREADS, Cfg::SMEM_BYTES, stream>>>(ma, mb, args);
     return cudaGetLastError();
@@ -583,12 +587,13 @@ cudaError_t launch_gemm_tn_pair(const void* A, int64_t lda, const void* B, int64
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
     const int pairs = std::min(a.num_tiles, dev->num_sms / 2);
-    static bool attr_set = false;
-    if (!attr_set) {
+    static bool attr_set[64] = {};
+    if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
+    if (!attr_set[dev->device]) {
         cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair_kernel,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, PAIR_SMEM_BYTES);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr_set[dev->device] = true;
     }
     tc_gemm_pair_kernel<<<2 * pairs, GEMM_THREADS, PAIR_SMEM_BYTES, stream>>>(ma, mb, a);
     return cudaGetLastError();

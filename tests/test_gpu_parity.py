@@ -55,7 +55,7 @@ def make_layer(K, M, N, seed, outliers=None, sigma=0.5):
 # ------------------------------------------------------------------------------ dense (Eq. 1)
 
 @pytest.mark.parametrize("N,K,M", [(128, 512, 512), (200, 520, 264), (1, 64, 8), (300, 1024, 776),
-                                   (129, 136, 392)])
+                                   (129, 136, 392), (9, 136, 392), (32, 520, 264), (5, 4096, 12288)])
 def test_dense_forward_matches_oracle(esp, N, K, M):
     _, X, W = make_layer(K, M, N, seed=100 + N)
     Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
@@ -102,6 +102,10 @@ FORWARD_CASES = [
     (8, 1024, 776, 448, 2),
     (8, 1024, 776, 448, 1),        # the same shape on both kernel families
     (5, 512, 512, 512, 0),         # full rank, automatic path
+    (17, 520, 264, 100, 2),        # decode kernel with 16- and 32-token groups, ragged
+    (32, 1024, 776, 448, 2),
+    (12, 512, 4104, 256, 2),       # M not a multiple of the 32-row tile
+    (32, 1024, 776, 448, 1),
 ]
 
 
