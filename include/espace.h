@@ -154,13 +154,22 @@ int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y
                           void* stream);
 
 /* As espace_linear_forward with the kernel family chosen by the caller:
- * path 0 = automatic, 1 = tensor-core kernels, 2 = small-N streaming kernels
- * (ESPACE_ERR_SHAPE if N or the layer is too large for the small-N kernels). */
-#define ESPACE_PATH_AUTO    0
-#define ESPACE_PATH_TENSOR  1
-#define ESPACE_PATH_SMALL_N 2
+ *   0 automatic;
+ *   1 tcgen05 tensor-core kernels: one persistent launch holding both products when N, L
+ *     and M exceed 128 (Z stays in L2 between them), else one launch per product;
+ *   2 the decode-shaped streaming kernel (ESPACE_ERR_SHAPE if N > 32 or the layer is too
+ *     large for it);
+ *   3 tcgen05 kernels, always one launch per product (Z through the scratch buffer). */
+#define ESPACE_PATH_AUTO         0
+#define ESPACE_PATH_TENSOR       1
+#define ESPACE_PATH_SMALL_N      2
+#define ESPACE_PATH_TENSOR_SPLIT 3
 int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev,
                                void* stream, int path);
+
+/* Number of kernel launches espace_linear_forward_path(p, ., N, ., ., path) makes (0 for
+ * N = 0), or -1 for invalid arguments or a path that cannot take N. Host-only query. */
+int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path);
 
 /* Capacity, in bf16 values, of the fixed scratch used by espace_linear_forward_noalloc:
  * 16 MiB, enough for N * Lp <= 8,388,608 (e.g. 4096 tokens at L = 2048). */

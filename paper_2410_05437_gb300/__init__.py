@@ -31,10 +31,11 @@ __all__ = [
     "espace_dense_forward",
     "espace_check", "espace_debug_wait_timeout", "espace_set_wait_limit_ns", "espace_set_phase_event",
     "espace_host_eigh",
-    "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "EXPORTED_SYMBOLS",
+    "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "PATH_TENSOR_SPLIT", "EXPORTED_SYMBOLS",
+    "espace_linear_forward_launches",
 ]
 
-PATH_AUTO, PATH_TENSOR, PATH_SMALL_N = 0, 1, 2
+PATH_AUTO, PATH_TENSOR, PATH_SMALL_N, PATH_TENSOR_SPLIT = 0, 1, 2, 3
 
 ERROR_NAMES = {1: "ARG", 2: "SHAPE", 3: "ALIGN", 4: "CUDA", 5: "TIMEOUT", 6: "STATE",
                7: "NOMEM", 8: "NUMERIC"}
@@ -84,6 +85,7 @@ _SIGNATURES = {
     "espace_linear_forward": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_linear_forward_path": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp, ctypes.c_int]),
     "espace_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
+    "espace_linear_forward_launches": (ctypes.c_int, [_vp, _i64, ctypes.c_int]),
     "espace_dense_forward": (ctypes.c_int, [_vp, _i64, _i64, _vp, _i64, _vp, _vp]),
     "espace_check": (ctypes.c_int, [_vp]),
     "espace_debug_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _vp]),
@@ -291,6 +293,10 @@ def espace_linear_forward_path(p: int, X, Y, path: int, N: int | None = None, st
     N = X.shape[0] if N is None else N
     _check(lib.espace_linear_forward_path(p, _dev_ptr(X), int(N), _dev_ptr(Y), _stream(stream),
                                           int(path)))
+
+
+def espace_linear_forward_launches(p: int, N: int, path: int = PATH_AUTO) -> int:
+    return lib.espace_linear_forward_launches(p, int(N), int(path))
 
 
 def espace_linear_forward_noalloc(p: int, X, Y, N: int | None = None, stream=None) -> None:

@@ -170,6 +170,7 @@ struct espace_proj_s {
     uint16_t* Z = nullptr;         // [zcap][Lp] bf16 scratch for the rank-L intermediate
     int64_t zcap = 0;
     unsigned int* bar = nullptr;   // grid barrier of the decode kernel (2 words, zeroed)
+    int* ready = nullptr;          // fused forward: 2 x ceil(zcap / 256) zeroed counters
     std::mutex mu;                 // guards Z growth
 };
 
@@ -547,10 +548,18 @@ void espace_proj_destroy(espace_proj_t p)
     if (p->WfT) cudaFree(p->WfT);
     if (p->Z) cudaFree(p->Z);
     if (p->bar) cudaFree(p->bar);
+    if (p->ready) cudaFree(p->ready);
     delete p;
 }
 
 // ---------------------------------------------------------------------------- forward
+
+// The fused kernel runs on CTA pairs with 256 x 256 tiles: worth it when both products
+// have more than one tile row and column.
+static bool fused_forward_applies(int n, int Lp, int M)
+{
+    return n > 128 && Lp > 128 && M > 128 && pair_kernel_enabled();
+}
 
 static int ensure_z(espace_proj_s* p, int64_t N, cudaStream_t st)
 {
@@ -558,10 +567,15 @@ static int ensure_z(espace_proj_s* p, int64_t N, cudaStream_t st)
     if (p->zcap >= N) return ESPACE_OK;
     CUDA_TRY(cudaStreamSynchronize(st), "forward: sync before scratch growth");
     if (p->Z) cudaFree(p->Z);
+    if (p->ready) cudaFree(p->ready);
     p->Z = nullptr;
+    p->ready = nullptr;
     p->zcap = 0;
     const int64_t cap = std::max<int64_t>(N, 128);
     cudaError_t e = cudaMalloc(&p->Z, sizeof(uint16_t) * cap * p->Lp);
+    const int64_t blocks = (cap + 255) / 256;
+    if (e == cudaSuccess) e = cudaMalloc(&p->ready, sizeof(int) * 2 * blocks);
+    if (e == cudaSuccess) e = cudaMemset(p->ready, 0, sizeof(int) * 2 * blocks);
     if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "forward: Z scratch of %lld tokens: %s", (long long)cap, cudaGetErrorString(e));
     p->zcap = cap;
     return ESPACE_OK;
@@ -576,7 +590,7 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
     if (X_dev == nullptr || Y_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward: null pointer");
     if (!aligned16(X_dev) || !aligned16(Y_dev)) return fail(ESPACE_ERR_ALIGN, "espace_linear_forward: X/Y not 16-byte aligned");
     if (N > (int64_t(1) << 31) - 256) return fail(ESPACE_ERR_SHAPE, "espace_linear_forward: N=%lld too large", (long long)N);
-    if (path < 0 || path > 2) return fail(ESPACE_ERR_ARG, "espace_linear_forward: unknown path %d", path);
+    if (path < 0 || path > 3) return fail(ESPACE_ERR_ARG, "espace_linear_forward: unknown path %d", path);
     const int K = static_cast<int>(p->K), M = static_cast<int>(p->M), Lp = static_cast<int>(p->Lp);
     const int n = static_cast<int>(N);
     DeviceInfo* dev = nullptr;
@@ -600,12 +614,35 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
         CUDA_TRY(launch_decode_forward(p->PT, p->WfT, X_dev, p->Z, Y_dev, K, Lp, M, n, p->bar, st),
                  "forward: decode kernel");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+    } else if (path != ESPACE_PATH_TENSOR_SPLIT && fused_forward_applies(n, Lp, M)) {
+        // one persistent launch holds both products; the phase event marks its start
+        if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+        CUDA_TRY(launch_forward_fused(X_dev, p->PT, p->Z, p->WfT, Y_dev, n, K, Lp, M, p->ready,
+                                      p->ready + (p->zcap + 255) / 256, st),
+                 "forward: fused kernel");
     } else {
         CUDA_TRY(launch_gemm_tn(X_dev, K, p->PT, K, n, Lp, K, p->Z, Lp, st), "forward: phase 1");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
         CUDA_TRY(launch_gemm_tn(p->Z, Lp, p->WfT, Lp, n, M, Lp, Y_dev, M, st), "forward: phase 2");
     }
     return ESPACE_OK;
+}
+
+int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path)
+{
+    if (p == nullptr || N < 0 || path < 0 || path > 3) return -1;
+    if (N == 0) return 0;
+    DeviceInfo* dev = nullptr;
+    {
+        DeviceGuard g(p->device);
+        if (device_info(&dev) != ESPACE_OK) return -1;
+    }
+    const int n = static_cast<int>(N), K = static_cast<int>(p->K), M = static_cast<int>(p->M),
+              Lp = static_cast<int>(p->Lp);
+    const bool small_ok = N <= DECODE_MAX_TOKENS && decode_supported(n, K, Lp, M, dev->num_sms);
+    if (path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok)) return small_ok ? 1 : -1;
+    if (path != ESPACE_PATH_TENSOR_SPLIT && fused_forward_applies(n, Lp, M)) return 1;
+    return 2;
 }
 
 int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev, void* stream)

@@ -24,6 +24,16 @@ uint64_t wait_limit_ns();
 cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
                            int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream);
 
+// The projected forward Z = X P, Y = Z W' in one persistent launch of the CTA-pair kernel:
+// Z tiles first, then Y tiles; a Y tile's producer waits (bounded) until the 256-row block
+// of Z it reads is complete. ready / done: ceil(N / 256) zeroed ints each, owned by the
+// caller, left zeroed again by the kernel. Needs N, Lp > 128 to be worthwhile.
+cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,
+                                 int K, int Lp, int M, int* ready, int* done, cudaStream_t stream);
+
+// Whether the CTA-pair kernels are enabled (ESPACE_DISABLE_PAIR_GEMM=1 turns them off).
+bool pair_kernel_enabled();
+
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
 

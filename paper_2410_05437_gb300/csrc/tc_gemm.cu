@@ -312,9 +312,74 @@ constexpr int PAIR_ACCS = 2;        // TMEM accumulators per CTA (1 or 2)
 constexpr int PAIR_TMEM_COLS = PAIR_ACCS * PAIR_BN;
 constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 256;
 
+// One product C[rows][cols] = A[rows][k] B[cols][k]^T of a pair program.
+struct PairProblem {
+    int rows, cols, kblocks, tiles_n, num_tiles;
+    void* out;
+    int64_t ldo;
+};
+
+// A program of one product, or of two where the second one's A operand is the first one's
+// output (the projected layer: Z = X P, then Y = Z W'). Row block tm of the second
+// product's A is read only after both CTAs of every tile in row block tm of the first
+// product have stored it: ready[tm] counts the epilogue warps that stored their rows
+// (target 8 x tiles_n of product 0: four warps in each of two CTAs per tile);
+// done[tm] counts the second product's producers that passed the check, and the last one
+// resets both, so the counters are zero again for the next launch.
+struct PairArgs {
+    PairProblem p[2];
+    int nprob;
+    int* ready;
+    int* done;
+    int* status;
+    uint64_t wait_limit_ns;
+};
+
+// Field-wise selection keeps the problem in registers (a dynamic index into the kernel
+// parameters would go through local memory).
+__device__ __forceinline__ PairProblem pair_problem_of(const PairArgs& a, int prob)
+{
+    PairProblem r;
+    r.rows = prob == 0 ? a.p[0].rows : a.p[1].rows;
+    r.cols = prob == 0 ? a.p[0].cols : a.p[1].cols;
+    r.kblocks = prob == 0 ? a.p[0].kblocks : a.p[1].kblocks;
+    r.tiles_n = prob == 0 ? a.p[0].tiles_n : a.p[1].tiles_n;
+    r.num_tiles = prob == 0 ? a.p[0].num_tiles : a.p[1].num_tiles;
+    r.out = prob == 0 ? a.p[0].out : a.p[1].out;
+    r.ldo = prob == 0 ? a.p[0].ldo : a.p[1].ldo;
+    return r;
+}
+
+__device__ __forceinline__ void pair_decode(const PairArgs& a, int item, int& prob, int& tm, int& tn)
+{
+    prob = item < a.p[0].num_tiles ? 0 : 1;
+    const int j = prob == 0 ? item : item - a.p[0].num_tiles;
+    const int tiles_n = prob == 0 ? a.p[0].tiles_n : a.p[1].tiles_n;
+    tm = j / tiles_n;
+    tn = j - tm * tiles_n;
+}
+
+__device__ __forceinline__ int ld_acquire_gpu(const int* p)
+{
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void red_release_gpu_add(int* p, int v)
+{
+    asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_global()
+{
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
-    tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a,
-                        const __grid_constant__ CUtensorMap map_b, const TcGemmArgs args)
+    tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_b0,
+                        const __grid_constant__ CUtensorMap map_a1, const __grid_constant__ CUtensorMap map_b1,
+                        const PairArgs args)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -349,8 +414,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
     }
     if (warp == 1) tmem_alloc_pair(tmem_slot, PAIR_TMEM_COLS);
     if (warp == 0 && lane == 0) {
-        tma_prefetch_map(&map_a);
-        tma_prefetch_map(&map_b);
+        tma_prefetch_map(&map_a0);
+        tma_prefetch_map(&map_b0);
+        if (args.nprob > 1) {
+            tma_prefetch_map(&map_a1);
+            tma_prefetch_map(&map_b1);
+        }
     }
     tc_fence_before_sync();
     cluster_sync();   // barriers of both CTAs initialised before any remote arrive or copy
@@ -362,7 +431,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
     const bool tmem_agree = peer_base == tmem_base;
     if (!tmem_agree && threadIdx.x == 0) atomicExch(args.status, ESPACE_ERR_STATE);
 
-    const int num_items = tmem_agree ? args.num_tiles : 0;
+    const int num_items =
+        tmem_agree ? args.p[0].num_tiles + (args.nprob > 1 ? args.p[1].num_tiles : 0) : 0;
     const uint64_t limit = args.wait_limit_ns;
 
     if (warp == 0) {
@@ -372,10 +442,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
             uint32_t phase = 0;
             bool ok = true;
             for (int item = pair; ok && item < num_items; item += npairs) {
-                const int tm = item / args.tiles_n, tn = item - (item / args.tiles_n) * args.tiles_n;
+                int prob, tm, tn;
+                pair_decode(args, item, prob, tm, tn);
+                const CUtensorMap* ma = prob == 0 ? &map_a0 : &map_a1;
+                const CUtensorMap* mb = prob == 0 ? &map_b0 : &map_b1;
+                if (prob == 1) {
+                    // row block tm of A (= product 0's output) must be complete: every
+                    // epilogue warp of both CTAs of every tile in it has signalled
+                    const int target = 2 * (EPI_THREADS / 32) * args.p[0].tiles_n;
+                    const uint64_t t0 = globaltimer_ns();
+                    uint32_t spins = 0;
+                    while (ld_acquire_gpu(args.ready + tm) < target) {
+                        if ((++spins & 15u) == 0 && (*abort_flag || globaltimer_ns() - t0 > limit)) {
+                            if (!*abort_flag) atomicExch(args.status, ESPACE_ERR_TIMEOUT);
+                            *abort_flag = 1;
+                            ok = false;
+                            break;
+                        }
+                        __nanosleep(128);
+                    }
+                    if (!ok) break;
+                    fence_proxy_async_global();   // the TMA reads below see those stores
+                    if (atomicAdd(args.done + tm, 1) == 2 * args.p[1].tiles_n - 1) {
+                        atomicExch(args.ready + tm, 0);
+                        atomicExch(args.done + tm, 0);
+                    }
+                }
                 const int row_a = tm * PAIR_BM + static_cast<int>(rank) * 128;
                 const int row_b = tn * PAIR_BN + static_cast<int>(rank) * 128;
-                for (int kb = 0; kb < args.kblocks; ++kb) {
+                const int kblocks = prob == 0 ? args.p[0].kblocks : args.p[1].kblocks;
+                for (int kb = 0; kb < kblocks; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
                         ok = false;
@@ -385,8 +481,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
                     uint8_t* sb = sa + PAIR_A_BYTES;
                     if (leader) mbar_arrive_expect_tx(&full[stage], 2 * PAIR_STAGE_BYTES);
                     const uint32_t bar = mapa_shared(smem_u32(&full[stage]), 0);
-                    tma_load_2d_pair(sa, &map_a, bar, kb * BK, row_a);
-                    tma_load_2d_pair(sb, &map_b, bar, kb * BK, row_b);
+                    tma_load_2d_pair(sa, ma, bar, kb * BK, row_a);
+                    tma_load_2d_pair(sb, mb, bar, kb * BK, row_b);
                     if (++stage == PAIR_STAGES) {
                         stage = 0;
                         phase ^= 1u;
@@ -405,12 +501,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
             uint32_t acc_phase = 0;
             bool ok = true;
             for (int item = pair; ok && item < num_items; item += npairs) {
+                int prob, tm, tn;
+                pair_decode(args, item, prob, tm, tn);
                 if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, args.status, limit,
                                ESPACE_ERR_TIMEOUT))
                     break;
                 tc_fence_after_sync();
                 const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * PAIR_BN);
-                for (int kb = 0; kb < args.kblocks; ++kb) {
+                const int kblocks = prob == 0 ? args.p[0].kblocks : args.p[1].kblocks;
+                for (int kb = 0; kb < kblocks; ++kb) {
                     if (!mbar_wait(&full[stage], phase, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
                         ok = false;
@@ -449,7 +548,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int item = pair; item < num_items; item += npairs) {
-            const int tm = item / args.tiles_n, tn = item - (item / args.tiles_n) * args.tiles_n;
+            int prob, tm, tn;
+            pair_decode(args, item, prob, tm, tn);
+            const PairProblem pb = pair_problem_of(args, prob);
             if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, args.status, limit,
                            ESPACE_ERR_TIMEOUT))
                 break;
@@ -458,16 +559,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
             const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                    static_cast<uint32_t>(acc * PAIR_BN);
             __nv_bfloat16* out_row =
-                reinterpret_cast<__nv_bfloat16*>(args.out) + static_cast<int64_t>(row) * args.ldo;
+                reinterpret_cast<__nv_bfloat16*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
 #pragma unroll 1
             for (int c = 0; c < PAIR_BN; c += 32) {
                 const int col0 = tn * PAIR_BN + c;
-                if (col0 >= args.cols) break;        // uniform across the warp
+                if (col0 >= pb.cols) break;          // uniform across the warp
                 uint32_t v[32];
                 tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
                 tmem_ld_wait();
-                if (row >= args.rows) continue;
-                if (col0 + 32 <= args.cols) {
+                if (row >= pb.rows) continue;
+                if (col0 + 32 <= pb.cols) {
                     uint4* dst = reinterpret_cast<uint4*>(out_row + col0);
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
@@ -481,7 +582,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
                 } else {
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
-                        if (col0 + i < args.cols)
+                        if (col0 + i < pb.cols)
                             out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
                 }
             }
@@ -490,6 +591,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
             if (++acc == PAIR_ACCS) {
                 acc = 0;
                 acc_phase ^= 1u;
+            }
+            if (prob == 0 && args.nprob > 1) {
+                // publish this warp's 32 rows of the tile to the second product's producers
+                // (per warp, so that no block-wide barrier can wait on a warp that gave up)
+                fence_proxy_async_global();
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) red_release_gpu_add(args.ready + tm, 1);
             }
         }
     }
@@ -565,28 +674,23 @@ cudaError_t launch_kernel(const CUtensorMap& ma, const CUtensorMap& mb, const Tc
     return cudaGetLastError();
 }
 
-// 256 x 256 tiles on CTA pairs; grid = 2 x min(tiles, SMs / 2).
-cudaError_t launch_gemm_tn_pair(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
-                                int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream,
-                                const DeviceInfo* dev)
+PairProblem pair_problem(int rows, int cols, int kdim, void* out, int64_t ldo)
 {
-    CUtensorMap ma, mb;
-    if (!encode_map(&ma, A, kdim, rows, lda, BK, 128)) return cudaErrorInvalidValue;
-    if (!encode_map(&mb, B, kdim, cols, ldb, BK, 128)) return cudaErrorInvalidValue;
-    TcGemmArgs a{};
-    a.rows = rows;
-    a.cols = cols;
-    a.kblocks = (kdim + BK - 1) / BK;
-    a.tiles_n = (cols + PAIR_BN - 1) / PAIR_BN;
-    a.num_tiles = ((rows + PAIR_BM - 1) / PAIR_BM) * a.tiles_n;
-    a.ksplit = 1;
-    a.kb_per_split = a.kblocks;
-    a.tile_list = nullptr;
-    a.out = C;
-    a.ldo = ldc;
-    a.status = dev->status;
-    a.wait_limit_ns = wait_limit_ns();
-    const int pairs = std::min(a.num_tiles, dev->num_sms / 2);
+    PairProblem p{};
+    p.rows = rows;
+    p.cols = cols;
+    p.kblocks = (kdim + BK - 1) / BK;
+    p.tiles_n = (cols + PAIR_BN - 1) / PAIR_BN;
+    p.num_tiles = ((rows + PAIR_BM - 1) / PAIR_BM) * p.tiles_n;
+    p.out = out;
+    p.ldo = ldo;
+    return p;
+}
+
+cudaError_t launch_pair(const CUtensorMap* maps, PairArgs& a, const DeviceInfo* dev, cudaStream_t stream)
+{
+    const int items = a.p[0].num_tiles + (a.nprob > 1 ? a.p[1].num_tiles : 0);
+    const int pairs = std::min(items, dev->num_sms / 2);
     static bool attr_set[64] = {};
     if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
     if (!attr_set[dev->device]) {
@@ -595,9 +699,29 @@ cudaError_t launch_gemm_tn_pair(const void* A, int64_t lda, const void* B, int64
         if (e != cudaSuccess) return e;
         attr_set[dev->device] = true;
     }
-    tc_gemm_pair_kernel<<<2 * pairs, GEMM_THREADS, PAIR_SMEM_BYTES, stream>>>(ma, mb, a);
+    tc_gemm_pair_kernel<<<2 * pairs, GEMM_THREADS, PAIR_SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
     return cudaGetLastError();
 }
+
+// 256 x 256 tiles on CTA pairs; grid = 2 x min(tiles, SMs / 2).
+cudaError_t launch_gemm_tn_pair(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
+                                int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream,
+                                const DeviceInfo* dev)
+{
+    CUtensorMap maps[4];
+    if (!encode_map(&maps[0], A, kdim, rows, lda, BK, 128)) return cudaErrorInvalidValue;
+    if (!encode_map(&maps[1], B, kdim, cols, ldb, BK, 128)) return cudaErrorInvalidValue;
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+    PairArgs a{};
+    a.p[0] = pair_problem(rows, cols, kdim, C, ldc);
+    a.nprob = 1;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return launch_pair(maps, a, dev, stream);
+}
+
+}  // namespace
 
 // The CTA-pair kernel is used unless ESPACE_DISABLE_PAIR_GEMM=1 is set in the environment.
 bool pair_kernel_enabled()
@@ -608,8 +732,6 @@ bool pair_kernel_enabled()
     }();
     return enabled;
 }
-
-}  // namespace
 
 cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ldb, int rows,
                            int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream)
@@ -716,6 +838,28 @@ cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStr
     a.wait_limit_ns = wait_limit_ns();
     const int grid = std::min(a.num_tiles * a.ksplit, dev->num_sms);
     return launch_kernel<256, 4, true, EPI_ATOMIC_UPPER_F32>(mx, mx, a, grid, stream);
+}
+
+cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,
+                                 int K, int Lp, int M, int* ready, int* done, cudaStream_t stream)
+{
+    if (N <= 0) return cudaSuccess;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    if (dev->num_sms < 2) return cudaErrorInvalidConfiguration;
+    CUtensorMap maps[4];
+    if (!encode_map(&maps[0], X, K, N, K, BK, 128) || !encode_map(&maps[1], PT, K, Lp, K, BK, 128) ||
+        !encode_map(&maps[2], Z, Lp, N, Lp, BK, 128) || !encode_map(&maps[3], WfT, Lp, M, Lp, BK, 128))
+        return cudaErrorInvalidValue;
+    PairArgs a{};
+    a.p[0] = pair_problem(N, Lp, K, Z, Lp);
+    a.p[1] = pair_problem(N, M, Lp, Y, M);
+    a.nprob = 2;
+    a.ready = ready;
+    a.done = done;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return launch_pair(maps, a, dev, stream);
 }
 
 }  // namespace espace

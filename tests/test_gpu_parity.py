@@ -106,7 +106,26 @@ FORWARD_CASES = [
     (32, 1024, 776, 448, 2),
     (12, 512, 4104, 256, 2),       # M not a multiple of the 32-row tile
     (32, 1024, 776, 448, 1),
+    (600, 1024, 1000, 512, 1),     # one persistent launch for both products, ragged M
+    (600, 1024, 1000, 512, 3),     # the same on two launches
+    (1000, 2048, 2312, 1000, 1),   # fused, ragged N / L / M, several row blocks
+    (300, 1024, 3000, 300, 3),
 ]
+
+
+def test_launch_counts(esp):
+    K, M, L = 1024, 1000, 512
+    P = synth.random_projection(K, L, seed=2)
+    p = esp.espace_proj_from_host(P, dev(synth.weights(M, K, seed=2)))
+    try:
+        assert esp.espace_linear_forward_launches(p, 0) == 0
+        assert esp.espace_linear_forward_launches(p, 1) == 1          # decode kernel
+        assert esp.espace_linear_forward_launches(p, 600) == 1        # fused
+        assert esp.espace_linear_forward_launches(p, 600, esp.PATH_TENSOR_SPLIT) == 2
+        assert esp.espace_linear_forward_launches(p, 100, esp.PATH_TENSOR) == 2
+        assert esp.espace_linear_forward_launches(p, 64, esp.PATH_SMALL_N) == -1
+    finally:
+        esp.espace_proj_destroy(p)
 
 
 @pytest.mark.parametrize("N,K,M,L,path", FORWARD_CASES)
