@@ -314,7 +314,11 @@ constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 256;
 
 // One product C[rows][cols] = A[rows][k] B[cols][k]^T of a pair program.
 struct PairProblem {
-    int rows, cols, kblocks, tiles_n, num_tiles;
+    int rows, cols, kblocks, tiles_n;
+    int num_tiles;           // output tiles
+    int ksplit;              // reduction splits per tile (work items = num_tiles * ksplit)
+    int kb_per_split;
+    const int2* tile_list;   // (tile row, tile col) pairs, or nullptr for the full grid
     void* out;
     int64_t ldo;
 };
@@ -345,18 +349,35 @@ __device__ __forceinline__ PairProblem pair_problem_of(const PairArgs& a, int pr
     r.kblocks = prob == 0 ? a.p[0].kblocks : a.p[1].kblocks;
     r.tiles_n = prob == 0 ? a.p[0].tiles_n : a.p[1].tiles_n;
     r.num_tiles = prob == 0 ? a.p[0].num_tiles : a.p[1].num_tiles;
+    r.ksplit = prob == 0 ? a.p[0].ksplit : a.p[1].ksplit;
+    r.kb_per_split = prob == 0 ? a.p[0].kb_per_split : a.p[1].kb_per_split;
+    r.tile_list = prob == 0 ? a.p[0].tile_list : a.p[1].tile_list;
     r.out = prob == 0 ? a.p[0].out : a.p[1].out;
     r.ldo = prob == 0 ? a.p[0].ldo : a.p[1].ldo;
     return r;
 }
 
-__device__ __forceinline__ void pair_decode(const PairArgs& a, int item, int& prob, int& tm, int& tn)
+__device__ __forceinline__ int pair_items(const PairProblem& p) { return p.num_tiles * p.ksplit; }
+
+// Work item -> (problem, tile row, tile column, k-block range).
+__device__ __forceinline__ void pair_decode(const PairArgs& a, int item, int& prob, int& tm, int& tn,
+                                            int& kb0, int& kb1)
 {
-    prob = item < a.p[0].num_tiles ? 0 : 1;
-    const int j = prob == 0 ? item : item - a.p[0].num_tiles;
-    const int tiles_n = prob == 0 ? a.p[0].tiles_n : a.p[1].tiles_n;
-    tm = j / tiles_n;
-    tn = j - tm * tiles_n;
+    const int n0 = a.p[0].num_tiles * a.p[0].ksplit;
+    prob = item < n0 ? 0 : 1;
+    const PairProblem p = pair_problem_of(a, prob);
+    const int j = prob == 0 ? item : item - n0;
+    const int tile = j / p.ksplit, split = j - tile * p.ksplit;
+    if (p.tile_list != nullptr) {
+        const int2 t = p.tile_list[tile];
+        tm = t.x;
+        tn = t.y;
+    } else {
+        tm = tile / p.tiles_n;
+        tn = tile - tm * p.tiles_n;
+    }
+    kb0 = split * p.kb_per_split;
+    kb1 = min(kb0 + p.kb_per_split, p.kblocks);
 }
 
 __device__ __forceinline__ int ld_acquire_gpu(const int* p)
@@ -376,6 +397,11 @@ __device__ __forceinline__ void fence_proxy_async_global()
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// SYRK = false: K-major operands, bf16 stores (the products of Eq. 3 and Eq. 1).
+// SYRK = true: both operands are one token-major X read M/N-major (64 features x 64 tokens
+// per box, two boxes per operand and CTA), and the epilogue adds each tile's upper triangle
+// (column >= row) to the fp32 sum S with atomics (Eq. 4).
+template <bool SYRK>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_b0,
                         const __grid_constant__ CUtensorMap map_a1, const __grid_constant__ CUtensorMap map_b1,
@@ -432,7 +458,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
     if (!tmem_agree && threadIdx.x == 0) atomicExch(args.status, ESPACE_ERR_STATE);
 
     const int num_items =
-        tmem_agree ? args.p[0].num_tiles + (args.nprob > 1 ? args.p[1].num_tiles : 0) : 0;
+        tmem_agree ? pair_items(args.p[0]) + (args.nprob > 1 ? pair_items(args.p[1]) : 0) : 0;
     const uint64_t limit = args.wait_limit_ns;
 
     if (warp == 0) {
@@ -442,8 +468,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
             uint32_t phase = 0;
             bool ok = true;
             for (int item = pair; ok && item < num_items; item += npairs) {
-                int prob, tm, tn;
-                pair_decode(args, item, prob, tm, tn);
+                int prob, tm, tn, kb0, kb1;
+                pair_decode(args, item, prob, tm, tn, kb0, kb1);
                 const CUtensorMap* ma = prob == 0 ? &map_a0 : &map_a1;
                 const CUtensorMap* mb = prob == 0 ? &map_b0 : &map_b1;
                 if (prob == 1) {
@@ -470,8 +496,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
                 }
                 const int row_a = tm * PAIR_BM + static_cast<int>(rank) * 128;
                 const int row_b = tn * PAIR_BN + static_cast<int>(rank) * 128;
-                const int kblocks = prob == 0 ? args.p[0].kblocks : args.p[1].kblocks;
-                for (int kb = 0; kb < kblocks; ++kb) {
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
                         ok = false;
@@ -481,8 +506,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
                     uint8_t* sb = sa + PAIR_A_BYTES;
                     if (leader) mbar_arrive_expect_tx(&full[stage], 2 * PAIR_STAGE_BYTES);
                     const uint32_t bar = mapa_shared(smem_u32(&full[stage]), 0);
-                    tma_load_2d_pair(sa, ma, bar, kb * BK, row_a);
-                    tma_load_2d_pair(sb, mb, bar, kb * BK, row_b);
+                    if (SYRK) {
+                        // 64 features x 64 tokens per box; the second 64 features at +8 KB
+                        tma_load_2d_pair(sa, ma, bar, row_a, kb * BK);
+                        tma_load_2d_pair(sa + 8192, ma, bar, row_a + 64, kb * BK);
+                        tma_load_2d_pair(sb, mb, bar, row_b, kb * BK);
+                        tma_load_2d_pair(sb + 8192, mb, bar, row_b + 64, kb * BK);
+                    } else {
+                        tma_load_2d_pair(sa, ma, bar, kb * BK, row_a);
+                        tma_load_2d_pair(sb, mb, bar, kb * BK, row_b);
+                    }
                     if (++stage == PAIR_STAGES) {
                         stage = 0;
                         phase ^= 1u;
@@ -494,22 +527,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer (leader)
         if (lane == 0 && leader) {
-            constexpr uint32_t idesc = idesc_bf16_f32(PAIR_BM, PAIR_BN, false, false);
+            constexpr uint32_t idesc = idesc_bf16_f32(PAIR_BM, PAIR_BN, SYRK, SYRK);
+            // K-major: the next 16-element K slice starts 32 bytes along the swizzled row;
+            // M/N-major: 16 tokens further = 16 rows of 128 bytes, 64-feature atoms 8 KB apart
+            constexpr uint32_t k_step = SYRK ? 2048u : 32u;
+            constexpr uint32_t lbo = SYRK ? 8192u : 16u;
             int stage = 0;
             uint32_t phase = 0;
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
             for (int item = pair; ok && item < num_items; item += npairs) {
-                int prob, tm, tn;
-                pair_decode(args, item, prob, tm, tn);
+                int prob, tm, tn, kb0, kb1;
+                pair_decode(args, item, prob, tm, tn, kb0, kb1);
                 if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, args.status, limit,
                                ESPACE_ERR_TIMEOUT))
                     break;
                 tc_fence_after_sync();
                 const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * PAIR_BN);
-                const int kblocks = prob == 0 ? args.p[0].kblocks : args.p[1].kblocks;
-                for (int kb = 0; kb < kblocks; ++kb) {
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(&full[stage], phase, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
                         ok = false;
@@ -520,9 +556,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
                     const uint32_t b_addr = a_addr + PAIR_A_BYTES;
 #pragma unroll
                     for (int j = 0; j < BK / UMMA_K; ++j) {
-                        const uint64_t ad = smem_desc_sw128(a_addr + j * 32, 16, 1024);
-                        const uint64_t bd = smem_desc_sw128(b_addr + j * 32, 16, 1024);
-                        umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > 0 || j > 0) ? 1u : 0u);
+                        const uint64_t ad = smem_desc_sw128(a_addr + j * k_step, lbo, 1024);
+                        const uint64_t bd = smem_desc_sw128(b_addr + j * k_step, lbo, 1024);
+                        umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > kb0 || j > 0) ? 1u : 0u);
                     }
                     umma_commit_pair(&empty[stage], 0x3);   // frees the stage in both CTAs
                     if (++stage == PAIR_STAGES) {
@@ -548,8 +584,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int item = pair; item < num_items; item += npairs) {
-            int prob, tm, tn;
-            pair_decode(args, item, prob, tm, tn);
+            int prob, tm, tn, kb0, kb1;
+            pair_decode(args, item, prob, tm, tn, kb0, kb1);
             const PairProblem pb = pair_problem_of(args, prob);
             if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, args.status, limit,
                            ESPACE_ERR_TIMEOUT))
@@ -558,8 +594,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
             const int row = tm * PAIR_BM + row_in_tile;
             const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                    static_cast<uint32_t>(acc * PAIR_BN);
-            __nv_bfloat16* out_row =
-                reinterpret_cast<__nv_bfloat16*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
 #pragma unroll 1
             for (int c = 0; c < PAIR_BN; c += 32) {
                 const int col0 = tn * PAIR_BN + c;
@@ -568,6 +602,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
                 tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
                 tmem_ld_wait();
                 if (row >= pb.rows) continue;
+                if (SYRK) {
+                    float* s_row = reinterpret_cast<float*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const int col = col0 + i;
+                        if (col < pb.cols && col >= row) atomicAdd(s_row + col, __uint_as_float(v[i]));
+                    }
+                    continue;
+                }
+                __nv_bfloat16* out_row =
+                    reinterpret_cast<__nv_bfloat16*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
                 if (col0 + 32 <= pb.cols) {
                     uint4* dst = reinterpret_cast<uint4*>(out_row + col0);
 #pragma unroll
@@ -682,24 +727,28 @@ PairProblem pair_problem(int rows, int cols, int kdim, void* out, int64_t ldo)
     p.kblocks = (kdim + BK - 1) / BK;
     p.tiles_n = (cols + PAIR_BN - 1) / PAIR_BN;
     p.num_tiles = ((rows + PAIR_BM - 1) / PAIR_BM) * p.tiles_n;
+    p.ksplit = 1;
+    p.kb_per_split = p.kblocks;
+    p.tile_list = nullptr;
     p.out = out;
     p.ldo = ldo;
     return p;
 }
 
+template <bool SYRK>
 cudaError_t launch_pair(const CUtensorMap* maps, PairArgs& a, const DeviceInfo* dev, cudaStream_t stream)
 {
-    const int items = a.p[0].num_tiles + (a.nprob > 1 ? a.p[1].num_tiles : 0);
+    const int items = a.p[0].num_tiles * a.p[0].ksplit + (a.nprob > 1 ? a.p[1].num_tiles * a.p[1].ksplit : 0);
     const int pairs = std::min(items, dev->num_sms / 2);
+    auto kern = tc_gemm_pair_kernel<SYRK>;
     static bool attr_set[64] = {};
     if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
     if (!attr_set[dev->device]) {
-        cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, PAIR_SMEM_BYTES);
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, PAIR_SMEM_BYTES);
         if (e != cudaSuccess) return e;
         attr_set[dev->device] = true;
     }
-    tc_gemm_pair_kernel<<<2 * pairs, GEMM_THREADS, PAIR_SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
+    kern<<<2 * pairs, GEMM_THREADS, PAIR_SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
     return cudaGetLastError();
 }
 
@@ -718,7 +767,7 @@ cudaError_t launch_gemm_tn_pair(const void* A, int64_t lda, const void* B, int64
     a.nprob = 1;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
-    return launch_pair(maps, a, dev, stream);
+    return launch_pair<false>(maps, a, dev, stream);
 }
 
 }  // namespace
@@ -772,38 +821,56 @@ struct TileList {
     int count = 0;
 };
 
-// Upper-triangle tile pairs (128-row block, 256-column block) for one K, kept per device.
-int2* syrk_tiles(int K, int* count)
+// Upper-triangle tile pairs for one K and tile shape (rows x cols), kept per device.
+int2* syrk_tiles(int K, int tile_rows, int tile_cols, int* count)
 {
     static std::mutex mu;
-    static std::vector<std::pair<int, TileList>> cache;   // (device, list)
+    struct Entry {
+        int device, K, tr, tc;
+        TileList list;
+    };
+    static std::vector<Entry> cache;
     int device = 0;
     cudaGetDevice(&device);
     std::lock_guard<std::mutex> lock(mu);
     for (auto& e : cache)
-        if (e.first == device && e.second.K == K) {
-            *count = e.second.count;
-            return e.second.dev;
+        if (e.device == device && e.K == K && e.tr == tile_rows && e.tc == tile_cols) {
+            *count = e.list.count;
+            return e.list.dev;
         }
     std::vector<int2> host;
-    const int tm_n = (K + BM - 1) / BM, tn_n = (K + 255) / 256;
+    const int tm_n = (K + tile_rows - 1) / tile_rows, tn_n = (K + tile_cols - 1) / tile_cols;
     for (int tm = 0; tm < tm_n; ++tm)
         for (int tn = 0; tn < tn_n; ++tn)
-            if (tn * 256 + 255 >= tm * BM) host.push_back(make_int2(tm, tn));
+            if (tn * tile_cols + tile_cols - 1 >= tm * tile_rows) host.push_back(make_int2(tm, tn));
     int2* dev = nullptr;
     if (cudaMalloc(&dev, host.size() * sizeof(int2)) != cudaSuccess) return nullptr;
-    if (cudaMemcpy(dev, host.data(), host.size() * sizeof(int2), cudaMemcpyHostToDevice) !=
-        cudaSuccess) {
+    if (cudaMemcpy(dev, host.data(), host.size() * sizeof(int2), cudaMemcpyHostToDevice) != cudaSuccess) {
         cudaFree(dev);
         return nullptr;
     }
-    TileList t;
-    t.K = K;
-    t.dev = dev;
-    t.count = static_cast<int>(host.size());
-    cache.emplace_back(device, t);
-    *count = t.count;
+    Entry e;
+    e.device = device;
+    e.K = K;
+    e.tr = tile_rows;
+    e.tc = tile_cols;
+    e.list.K = K;
+    e.list.dev = dev;
+    e.list.count = static_cast<int>(host.size());
+    cache.push_back(e);
+    *count = e.list.count;
     return dev;
+}
+
+// Token splits so that there are about two work items per worker, at least 16 k-blocks
+// (1024 tokens) per split.
+void choose_splits(int kblocks, int tiles, int workers, int* ksplit, int* kb_per_split)
+{
+    const int want = std::max(1, (2 * workers + tiles - 1) / tiles);
+    int kbps = std::max(16, (kblocks + want - 1) / want);
+    kbps = std::min(kbps, kblocks);
+    *kb_per_split = kbps;
+    *ksplit = (kblocks + kbps - 1) / kbps;
 }
 
 }  // namespace
@@ -813,24 +880,43 @@ cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStr
     if (N <= 0) return cudaSuccess;
     DeviceInfo* dev = nullptr;
     if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    const int kblocks = static_cast<int>((N + BK - 1) / BK);
+    if (K > 128 && dev->num_sms >= 2 && pair_kernel_enabled()) {
+        // 256 x 256 upper-triangle tiles on CTA pairs
+        int count = 0;
+        const int2* tiles = syrk_tiles(K, PAIR_BM, PAIR_BN, &count);
+        if (tiles == nullptr) return cudaErrorMemoryAllocation;
+        CUtensorMap maps[4];
+        if (!encode_map(&maps[0], X, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
+        maps[1] = maps[2] = maps[3] = maps[0];
+        PairArgs a{};
+        PairProblem& p = a.p[0];
+        p.rows = K;
+        p.cols = K;
+        p.kblocks = kblocks;
+        p.tiles_n = 0;
+        p.num_tiles = count;
+        choose_splits(kblocks, count, dev->num_sms / 2, &p.ksplit, &p.kb_per_split);
+        p.tile_list = tiles;
+        p.out = S;
+        p.ldo = K;
+        a.nprob = 1;
+        a.status = dev->status;
+        a.wait_limit_ns = wait_limit_ns();
+        return launch_pair<true>(maps, a, dev, stream);
+    }
     int count = 0;
-    const int2* tiles = syrk_tiles(K, &count);
+    const int2* tiles = syrk_tiles(K, BM, 256, &count);
     if (tiles == nullptr) return cudaErrorMemoryAllocation;
     CUtensorMap mx;
     if (!encode_map(&mx, X, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
     TcGemmArgs a{};
     a.rows = K;
     a.cols = K;
-    a.kblocks = static_cast<int>((N + BK - 1) / BK);
+    a.kblocks = kblocks;
     a.tiles_n = 0;
     a.num_tiles = count;
-    // split the tokens so that there are about two work items per SM, at least 16 blocks
-    // (1024 tokens) per split
-    int want_splits = std::max(1, (2 * dev->num_sms + count - 1) / count);
-    int kbps = std::max(16, (a.kblocks + want_splits - 1) / want_splits);
-    kbps = std::min(kbps, a.kblocks);
-    a.kb_per_split = kbps;
-    a.ksplit = (a.kblocks + kbps - 1) / kbps;
+    choose_splits(kblocks, count, dev->num_sms, &a.ksplit, &a.kb_per_split);
     a.tile_list = tiles;
     a.out = S;
     a.ldo = K;
@@ -859,7 +945,7 @@ cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const v
     a.done = done;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
-    return launch_pair(maps, a, dev, stream);
+    return launch_pair<false>(maps, a, dev, stream);
 }
 
 }  // namespace espace
