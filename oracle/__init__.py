@@ -7,6 +7,7 @@ C file ``espace_oracle.c`` (built by ``oracle.build``); this module only marshal
 arrays and chains the steps in the order the paper states them:
 
 * ``autocorr_sum``      Eq. 4, the sum of x x^T over calibration tokens (no centering);
+* ``autocorr_rows``     the same for selected rows (large K);
 * ``eigh``              the EVD of Sec. 3.1 by cyclic Jacobi, eigenvalues decreasing;
 * ``build_projection``  Thm. 1: P = the L principal eigenvectors of C = S / n, then bf16;
 * ``fold``              W' = P^T W (Sec. 2.2), bf16;
@@ -46,6 +47,7 @@ def _load():
         lib.oracle_bf16_round_array.argtypes = [_dp, _i64]
         lib.oracle_autocorr_sum.argtypes = [_dp, _i64, _i64, _dp]
         lib.oracle_autocorr_normalized_sum.argtypes = [_dp, _i64, _i64, _dp]
+        lib.oracle_autocorr_rows.argtypes = [_dp, _i64, _i64, ctypes.POINTER(ctypes.c_int64), _i64, _dp]
         lib.oracle_jacobi_eigh.restype = ctypes.c_int
         lib.oracle_jacobi_eigh.argtypes = [_dp, _i64, _dp, _dp, ctypes.c_int, ctypes.c_double]
         lib.oracle_fold.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp, ctypes.c_int]
@@ -80,6 +82,16 @@ def autocorr_sum(X, S: np.ndarray | None = None) -> np.ndarray:
     n, K = X.shape
     S = np.zeros((K, K)) if S is None else _f64(S).copy()
     _load().oracle_autocorr_sum(_ptr(X), n, K, _ptr(S))
+    return S
+
+
+def autocorr_rows(X, rows) -> np.ndarray:
+    """Eq. 4 for the listed rows only: ``sum_t x_t[rows] x_t^T`` as ``[len(rows), K]``."""
+    X = _f64(X)
+    n, K = X.shape
+    r = np.ascontiguousarray(np.asarray(rows, dtype=np.int64))
+    S = np.zeros((len(r), K))
+    _load().oracle_autocorr_rows(_ptr(X), n, K, r.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), len(r), _ptr(S))
     return S
 
 

@@ -11,6 +11,7 @@
  *
  *   oracle_bf16_round        rounding of a real number to the nearest bf16 value
  *   oracle_autocorr_sum      S += sum_t x_t x_t^T                      (Sec. 3.1, Eq. 4)
+ *   oracle_autocorr_rows     the same for selected rows of S            (Sec. 3.1, Eq. 4)
  *   oracle_jacobi_eigh       C = V D V^T, eigenvalues sorted decreasing (Sec. 3.1, Thm. 1)
  *   oracle_fold              W' = P^T W                                 (Sec. 2.2, Eq. 3)
  *   oracle_project           Z = P^T X (stored token-major as X P)      (Sec. 2.2, Eq. 3)
@@ -65,6 +66,21 @@ void oracle_autocorr_sum(const double* X, int64_t n, int64_t K, double* S)
         for (int64_t t = 0; t < n; ++t) {
             const double xi = X[t * K + i];
             for (int64_t j = 0; j < K; ++j) S[i * K + j] += xi * X[t * K + j];
+        }
+    }
+}
+
+/* Eq. 4 restricted to the rows listed in `rows` (nrows of them): S[r][j] += sum_t
+ * X[t][rows[r]] X[t][j], S being nrows x K. */
+void oracle_autocorr_rows(const double* X, int64_t n, int64_t K, const int64_t* rows, int64_t nrows,
+                          double* S)
+{
+    #pragma omp parallel for schedule(static)
+    for (int64_t r = 0; r < nrows; ++r) {
+        const int64_t i = rows[r];
+        for (int64_t t = 0; t < n; ++t) {
+            const double xi = X[t * K + i];
+            for (int64_t j = 0; j < K; ++j) S[r * K + j] += xi * X[t * K + j];
         }
     }
 }

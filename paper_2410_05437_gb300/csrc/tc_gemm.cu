@@ -311,6 +311,16 @@ constexpr int PAIR_STAGE_BYTES = PAIR_A_BYTES + PAIR_B_BYTES;
 constexpr int PAIR_ACCS = 2;        // TMEM accumulators per CTA (1 or 2)
 constexpr int PAIR_TMEM_COLS = PAIR_ACCS * PAIR_BN;
 constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 256;
+// The autocorrelation restarts its TMEM accumulator every SYRK_CHUNK k-blocks (1024
+// tokens) and its epilogue adds the chunks in fp32 registers, so that long token runs do
+// not lose precision in the tensor core's accumulator.
+constexpr int SYRK_CHUNK = 16;
+
+template <bool SYRK>
+struct PairShape {
+    static constexpr int EPI_WARPS = SYRK ? 8 : 4;   // SYRK: two warps per TMEM lane quarter
+    static constexpr int THREADS = 64 + 32 * EPI_WARPS;
+};
 
 // One product C[rows][cols] = A[rows][k] B[cols][k]^T of a pair program.
 struct PairProblem {
@@ -402,7 +412,7 @@ __device__ __forceinline__ void fence_proxy_async_global()
 // per box, two boxes per operand and CTA), and the epilogue adds each tile's upper triangle
 // (column >= row) to the fp32 sum S with atomics (Eq. 4).
 template <bool SYRK>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THREADS, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_b0,
                         const __grid_constant__ CUtensorMap map_a1, const __grid_constant__ CUtensorMap map_b1,
                         const PairArgs args)
@@ -432,7 +442,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 2 * EPI_THREADS);   // both CTAs' epilogue threads
+            mbar_init(&tempty[a], 2 * 32 * PairShape<SYRK>::EPI_WARPS);   // both CTAs' epilogues
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -540,42 +550,110 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
             for (int item = pair; ok && item < num_items; item += npairs) {
                 int prob, tm, tn, kb0, kb1;
                 pair_decode(args, item, prob, tm, tn, kb0, kb1);
-                if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, args.status, limit,
-                               ESPACE_ERR_TIMEOUT))
-                    break;
-                tc_fence_after_sync();
-                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * PAIR_BN);
-                for (int kb = kb0; kb < kb1; ++kb) {
-                    if (!mbar_wait(&full[stage], phase, abort_flag, args.status, limit,
+                // one accumulation per item, or per 16-block chunk of it for SYRK
+                const int chunk = SYRK ? SYRK_CHUNK : (kb1 - kb0);
+                for (int c0 = kb0; ok && c0 < kb1; c0 += chunk) {
+                    const int c1 = min(c0 + chunk, kb1);
+                    if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after_sync();
-                    const uint32_t a_addr = smem_u32(smem + stage * PAIR_STAGE_BYTES);
-                    const uint32_t b_addr = a_addr + PAIR_A_BYTES;
+                    const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * PAIR_BN);
+                    for (int kb = c0; kb < c1; ++kb) {
+                        if (!mbar_wait(&full[stage], phase, abort_flag, args.status, limit,
+                                       ESPACE_ERR_TIMEOUT)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after_sync();
+                        const uint32_t a_addr = smem_u32(smem + stage * PAIR_STAGE_BYTES);
+                        const uint32_t b_addr = a_addr + PAIR_A_BYTES;
 #pragma unroll
-                    for (int j = 0; j < BK / UMMA_K; ++j) {
-                        const uint64_t ad = smem_desc_sw128(a_addr + j * k_step, lbo, 1024);
-                        const uint64_t bd = smem_desc_sw128(b_addr + j * k_step, lbo, 1024);
-                        umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > kb0 || j > 0) ? 1u : 0u);
+                        for (int j = 0; j < BK / UMMA_K; ++j) {
+                            const uint64_t ad = smem_desc_sw128(a_addr + j * k_step, lbo, 1024);
+                            const uint64_t bd = smem_desc_sw128(b_addr + j * k_step, lbo, 1024);
+                            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > c0 || j > 0) ? 1u : 0u);
+                        }
+                        umma_commit_pair(&empty[stage], 0x3);   // frees the stage in both CTAs
+                        if (++stage == PAIR_STAGES) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
                     }
-                    umma_commit_pair(&empty[stage], 0x3);   // frees the stage in both CTAs
-                    if (++stage == PAIR_STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
+                    if (!ok) break;
+                    umma_commit_pair(&tfull[acc], 0x3);          // both halves ready to drain
+                    if (++acc == PAIR_ACCS) {
+                        acc = 0;
+                        acc_phase ^= 1u;
                     }
-                }
-                if (!ok) break;
-                umma_commit_pair(&tfull[acc], 0x3);          // both halves ready to drain
-                if (++acc == PAIR_ACCS) {
-                    acc = 0;
-                    acc_phase ^= 1u;
                 }
             }
             umma_commit_pair(drain, 0x1);
             volatile int never = 0;
             mbar_wait(drain, 0, &never, args.status, limit, ESPACE_ERR_TIMEOUT);
+        }
+    } else if (SYRK) {
+        // ------------------------------------------------------------ SYRK epilogue (8 warps)
+        // warp pair (w, w + 4) shares a TMEM lane quarter and splits its 256 columns
+        const int ew = warp - 2;
+        const int quarter = warp & 3;
+        const int half = ew >> 2;
+        const int row_in_tile = static_cast<int>(rank) * 128 + quarter * 32 + lane;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        bool ok = true;
+        for (int item = pair; ok && item < num_items; item += npairs) {
+            int prob, tm, tn, kb0, kb1;
+            pair_decode(args, item, prob, tm, tn, kb0, kb1);
+            const PairProblem pb = pair_problem_of(args, prob);
+            float run[128];
+#pragma unroll
+            for (int i = 0; i < 128; ++i) run[i] = 0.f;
+            for (int c0 = kb0; c0 < kb1; c0 += SYRK_CHUNK) {
+                if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, args.status, limit,
+                               ESPACE_ERR_TIMEOUT)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after_sync();
+                const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                       static_cast<uint32_t>(acc * PAIR_BN + half * 128);
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    uint32_t v[16];
+                    tmem_ld_16cols(t_row + static_cast<uint32_t>(c * 16), v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) run[c * 16 + i] += __uint_as_float(v[i]);
+                }
+                tc_fence_before_sync();
+                mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[acc]), 0));
+                if (++acc == PAIR_ACCS) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+            // S[row][col] += run for the upper triangle (col >= row), 16 bytes at a time
+            const int row = tm * PAIR_BM + row_in_tile;
+            if (row < pb.rows) {
+                float* s_row = reinterpret_cast<float*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
+                const int colb = tn * PAIR_BN + half * 128;
+#pragma unroll
+                for (int i = 0; i < 128; i += 4) {
+                    const int col = colb + i;
+                    if (col >= row && col + 3 < pb.cols) {
+                        atomicAdd(reinterpret_cast<float4*>(s_row + col),
+                                  make_float4(run[i], run[i + 1], run[i + 2], run[i + 3]));
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 4; ++j)
+                            if (col + j >= row && col + j < pb.cols) atomicAdd(s_row + col + j, run[i + j]);
+                    }
+                }
+            }
         }
     } else {
         // ------------------------------------------------------------ epilogue (both CTAs)
@@ -602,15 +680,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(GEMM_THREADS, 1)
                 tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
                 tmem_ld_wait();
                 if (row >= pb.rows) continue;
-                if (SYRK) {
-                    float* s_row = reinterpret_cast<float*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const int col = col0 + i;
-                        if (col < pb.cols && col >= row) atomicAdd(s_row + col, __uint_as_float(v[i]));
-                    }
-                    continue;
-                }
                 __nv_bfloat16* out_row =
                     reinterpret_cast<__nv_bfloat16*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
                 if (col0 + 32 <= pb.cols) {
@@ -748,7 +817,7 @@ cudaError_t launch_pair(const CUtensorMap* maps, PairArgs& a, const DeviceInfo* 
         if (e != cudaSuccess) return e;
         attr_set[dev->device] = true;
     }
-    kern<<<2 * pairs, GEMM_THREADS, PAIR_SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
+    kern<<<2 * pairs, PairShape<SYRK>::THREADS, PAIR_SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
     return cudaGetLastError();
 }
 
@@ -916,7 +985,10 @@ cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStr
     a.kblocks = kblocks;
     a.tiles_n = 0;
     a.num_tiles = count;
-    choose_splits(kblocks, count, dev->num_sms, &a.ksplit, &a.kb_per_split);
+    // this kernel accumulates a whole split in TMEM: splits of at most 1024 tokens keep the
+    // fp32 accumulator precise (S is small whenever this path runs)
+    a.kb_per_split = std::min(SYRK_CHUNK, kblocks);
+    a.ksplit = (kblocks + a.kb_per_split - 1) / a.kb_per_split;
     a.tile_list = tiles;
     a.out = S;
     a.ldo = K;

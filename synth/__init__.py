@@ -173,6 +173,22 @@ def weights_device(M: int, K: int, seed: int = BASE_SEED, chunk: int = 0,
     return (w * (1.0 / math.sqrt(K))).to(torch.bfloat16)
 
 
+def structured_projection(K: int, L: int, seed: int = BASE_SEED) -> np.ndarray:
+    """A seeded ``K x L`` fp64 matrix with orthonormal columns built in O(K L): the first L
+    columns of (four Householder reflectors) x (signed permutation). Used at shapes where a
+    Gaussian QR would take minutes."""
+    rg = generator(seed, "projection", 1)
+    perm = rg.permutation(K)[:L]
+    signs = np.where(rg.random(L) < 0.5, -1.0, 1.0)
+    Q = np.zeros((K, L))
+    Q[perm, np.arange(L)] = signs
+    for _ in range(4):
+        v = rg.standard_normal(K)
+        v /= np.linalg.norm(v)
+        Q -= 2.0 * np.outer(v, v @ Q)
+    return Q
+
+
 def random_projection(K: int, L: int, seed: int = BASE_SEED) -> np.ndarray:
     """A seeded ``K x L`` fp64 matrix with orthonormal columns."""
     return haar_orthonormal(generator(seed, "projection"), K, L)

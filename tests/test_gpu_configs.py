@@ -1,0 +1,140 @@
+"""Parity at the full sizes of the benchmark's workloads, on sampled outputs.
+
+Each test runs the library on the whole layer (every token, every output, the launch
+configuration of the benchmark) and compares a seeded sample of outputs -- every output
+feature in a sample of columns, for a sample of tokens including the first and the last --
+with the fp64 oracle, which computes those outputs one by one. Tolerances as in
+test_gpu_parity.py.
+
+Workloads: the Llama2-7B MLP (gate+up K=4096 -> M=22016 and down K=11008 -> M=4096 with a
+silu(a)*b input) over a rank sweep; the GPT3-22B / Nemotron4 layer at 16,384 tokens (QKV,
+FC1, FC2 at L = K/2) and its calibration at K = 6144; and the decode-shaped token sweep
+N = 1 .. 512 on the Llama2-7B layers at L = K/2.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+Y_REL = 4e-3
+Y_MAX = 2e-2
+C_REL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def esp():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2410_05437_gb300 as esp
+    return esp
+
+
+def f64(t):
+    return synth.bf16_to_f64(t.cpu())
+
+
+def sampled_check(esp, X, W, P, n_tok, n_col, seed, path=0):
+    """Runs the whole layer on the GPU and checks sampled outputs against the oracle."""
+    N, K = X.shape
+    M = W.shape[0]
+    Wd = W.cuda()
+    p = esp.espace_proj_from_host(P, Wd)
+    try:
+        Xd = X.cuda()
+        Y = torch.full((N, M), float("nan"), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward_path(p, Xd, Y, path)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        del Xd, Wd
+        r = np.random.default_rng(seed)
+        toks = np.unique(np.concatenate([[0, N - 1], r.choice(N, min(n_tok, N), replace=False)]))
+        cols = np.sort(r.choice(M, min(n_col, M), replace=False))
+        Pb = oracle.bf16_round(P)
+        Wf_o = oracle.fold(Pb, f64(W[cols]))
+        Y_o = oracle.contract(oracle.project(f64(X[toks]), Pb), Wf_o)
+        Yg = f64(Y[toks][:, cols])
+        assert np.all(np.isfinite(Yg))
+        err = np.linalg.norm(Yg - Y_o) / np.linalg.norm(Y_o)
+        mx = np.abs(Yg - Y_o).max() / np.abs(Y_o).max()
+        assert err <= Y_REL, f"normwise {err:.3e}"
+        assert mx <= Y_MAX, f"max {mx:.3e}"
+        assert not torch.isnan(Y).any()
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+# ------------------------------------------------------------------ Llama2-7B MLP, rank sweep
+
+@pytest.mark.parametrize("frac", [0.8, 0.5])
+def test_llama2_gate_up(esp, frac):
+    K, M, N = 4096, 22016, 8192
+    L = int(round(frac * K))
+    seed = synth.config_seed("llama2_mlp_gate_up")
+    X = synth.ActivationModel(K, seed=seed).sample(N)
+    W = synth.weights(M, K, seed=seed)
+    P = synth.structured_projection(K, L, seed=seed)
+    sampled_check(esp, X, W, P, 24, 96, seed)
+
+
+@pytest.mark.parametrize("frac", [0.8, 0.5])
+def test_llama2_down_gated_input(esp, frac):
+    K, M, N = 11008, 4096, 8192
+    L = int(round(frac * K))
+    seed = synth.config_seed("llama2_mlp_down")
+    X = synth.ActivationModel(K, seed=seed).sample_gated(N)
+    W = synth.weights(M, K, seed=seed)
+    P = synth.structured_projection(K, L, seed=seed)
+    sampled_check(esp, X, W, P, 16, 64, seed)
+
+
+# ------------------------------------------------------------------ GPT3-22B / Nemotron4 layer
+
+@pytest.mark.parametrize("name", ["gpt3_22b_qkv", "gpt3_22b_fc1", "gpt3_22b_fc2"])
+def test_gpt3_22b_layer(esp, name):
+    cfg = synth.CONFIGS[name]
+    K, M, L, N = cfg["K"], cfg["M"], cfg["L"], cfg["N"]
+    seed = synth.config_seed(name)
+    X = synth.ActivationModel(K, seed=seed).sample(N)
+    W = synth.weights(M, K, seed=seed)
+    P = synth.structured_projection(K, L, seed=seed)
+    sampled_check(esp, X, W, P, 8, 48, seed)
+
+
+def test_gpt3_22b_calibration_rows(esp):
+    """C at K = 6144 after 16,384 tokens in two chunks: sampled rows against Eq. 4."""
+    K, n = 6144, 16384
+    seed = synth.config_seed("gpt3_22b_qkv")
+    X = synth.ActivationModel(K, seed=seed).sample(n, stream="calib_tokens")
+    h = esp.espace_calib_create(K)
+    try:
+        Xd = X.cuda()
+        esp.espace_calib_accumulate(h, Xd[: n // 2].contiguous())
+        esp.espace_calib_accumulate(h, Xd[n // 2:].contiguous())
+        C, cnt = esp.espace_calib_read(h, K)
+        esp.espace_check()
+        assert cnt == n
+        rows = np.sort(np.random.default_rng(seed).choice(K, 8, replace=False))
+        C_o = oracle.autocorr_rows(f64(X), rows) / n
+        err = np.linalg.norm(C[rows] - C_o) / np.linalg.norm(C_o)
+        assert err <= C_REL, f"C rows normwise {err:.3e}"
+    finally:
+        esp.espace_calib_destroy(h)
+
+
+# ------------------------------------------------------------------ decode-shaped token sweep
+
+@pytest.mark.parametrize("layer", ["qkv", "o", "gate_up", "down"])
+@pytest.mark.parametrize("N", synth.DECODE_TOKENS)
+def test_decode_sweep(esp, layer, N):
+    K, M = synth.DECODE_LAYERS[layer]
+    L = K // 2
+    seed = synth.BASE_SEED + 100 + N
+    model = synth.ActivationModel(K, seed=seed)
+    X = model.sample_gated(N) if layer == "down" else model.sample(N)
+    W = synth.weights(M, K, seed=seed)
+    P = synth.structured_projection(K, L, seed=seed)
+    sampled_check(esp, X, W, P, 16, 64, seed)

@@ -96,6 +96,18 @@ def test_autocorr_invariants():
     assert w.min() >= -1e-12 * w.max()
 
 
+def test_autocorr_rows_are_rows_of_the_full_sum():
+    r = rng(17)
+    X = r.standard_normal((40, 11))
+    rows = [0, 7, 3, 10]
+    assert np.allclose(oracle.autocorr_rows(X, rows), oracle.autocorr_sum(X)[rows], rtol=1e-13, atol=1e-13)
+
+
+def test_structured_projection_is_orthonormal():
+    P = synth.structured_projection(300, 120, seed=4)
+    assert np.allclose(P.T @ P, np.eye(120), atol=1e-12)
+
+
 def test_normalized_autocorr_is_autocorr_of_unit_vectors():
     r = rng(5)
     X = r.standard_normal((50, 9)) * 7.0
