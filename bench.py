@@ -40,6 +40,10 @@ METRIC = "ESPACE linear forward TFLOP/s (Llama2-7B QKV prefill, L=K/2)"
 UNIT = "TFLOP/s"
 SETS = 4
 
+# DRAM bytes (read + write) of one launch of the dominant kernel at this workload, from the
+# ncu capture summarized in profiles/fused_forward_llama2_qkv_prefill.md (same kernel build).
+FUSED_FORWARD_TRAFFIC_BYTES = 157095680 + 92755456
+
 
 def parse():
     ap = argparse.ArgumentParser()
@@ -48,6 +52,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-rows", action="store_true", help="skip the side measurements")
+    ap.add_argument("--profile-case", choices=["fused", "syrk", "decode"],
+                    help="run a few launches of one kernel on a small fixed case (for ncu) and exit")
     return ap.parse_args()
 
 
@@ -311,7 +317,9 @@ def run_ours(args, world, rank, local):
         "roofline": {"kernel": k_name, "bound": "tensor",
                      "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
                      "frac": achieved / peak_tc, "peak_kind": f"{peak_kind} bf16 burst",
-                     "flops_per_launch": k_flops, "ms_per_launch": k_ms, "traffic": None},
+                     "flops_per_launch": k_flops, "ms_per_launch": k_ms,
+                     "traffic": FUSED_FORWARD_TRAFFIC_BYTES if fused else None,
+                     "algorithmic_bytes": 2.0 * (N * K + K * L + L * M + N * M)},
         "phases_ms": {"before_event": statistics.mean(phase1), "after_event": statistics.mean(phase2),
                       "launches_per_step": 1 if fused else 2},
         "roofline_step": {"frac_of_tensor_peak": (flops / (ms_per_step * 1e-3) / 1e12) / peak_tc,
@@ -438,8 +446,40 @@ def graph_time_us(call, per_graph=20, replays=10):
     return a.elapsed_time(b) * 1e3 / (per_graph * replays)
 
 
+def profile_case(which):
+    """A few launches of one kernel, with little else on the GPU: the target of the ncu
+    captures summarized under profiles/ (launch 3 of the fused forward, launch 2 of the
+    calibration SYRK, launch 3 of the decode kernel)."""
+    import paper_2410_05437_gb300 as esp
+    torch.cuda.set_device(0)
+    if which in ("fused", "decode"):
+        K, M, L = 4096, 12288, 2048
+        N = 4096 if which == "fused" else 1
+        W = synth.weights_device(M, K)
+        p = esp.espace_proj_from_host(synth.random_projection(K, L), W)      # launch 1: fold
+        X = synth.ActivationModel(K).sample_device(N)
+        Y = torch.empty(N, M, device="cuda", dtype=torch.bfloat16)
+        for _ in range(3):
+            esp.espace_linear_forward(p, X, Y)
+        torch.cuda.synchronize()
+        esp.espace_proj_destroy(p)
+    else:
+        K, n = 4096, 65536
+        X = synth.ActivationModel(K).sample_device(n, stream="calib_tokens")
+        h = esp.espace_calib_create(K)
+        for _ in range(2):
+            esp.espace_calib_accumulate(h, X)
+        torch.cuda.synchronize()
+        esp.espace_calib_destroy(h)
+    esp.espace_check()
+    print(json.dumps({"profile_case": which, "ok": True}))
+
+
 def main():
     args = parse()
+    if args.profile_case:
+        profile_case(args.profile_case)
+        return
     world, rank, local = dist_init(args.gpus)
     if args.impl == "reference":
         run_reference(args, world, rank)
