@@ -2,27 +2,45 @@
 //
 // One cooperative launch computes both products of Eq. 3:
 //   phase 1  Z[n][l] = bf16( sum_k X[n][k] P^T[l][k] )   P^T streamed from HBM once
-//   -------  grid barrier (bounded spin) --------------------------------------------
+//   -------  grid barrier -------------------------------------------------------------
 //   phase 2  Y[n][m] = bf16( sum_l Z[n][l] W'^T[m][l] )  W'^T streamed once
 // (and, with one phase only, the dense decode product Y = X W^T).
 //
-// Streaming: at launch, each CTA asks the L2 to prefetch (cp.async.bulk.prefetch.L2, 64 KB
-// per request) the rows it will read in phase 2, so the HBM stays busy across the grid
-// barrier and phase 2 reads mostly from L2.
+// Streaming. Each CTA owns a contiguous range of rows of each streamed matrix; the ranges
+// are balanced over both phases together by bytes. One producer thread walks the CTA's
+// stages -- (up to 8 rows) x (a k-block of up to SK elements) -- in the order they are
+// consumed, phase 1 then phase 2, and copies each row piece into a ring of shared-memory
+// stages with 1-D bulk copies (cp.async.bulk) completing on the stage's mbarrier. The
+// producer does not wait for the grid barrier: while the consumers wait for Z, it keeps
+// filling the ring with W'^T rows, so HBM stays busy across the barrier.
 //
-// Compute: each CTA owns a contiguous range of 16-row blocks of the streamed matrix A; its
-// 16 warps split the reduction dimension into 16 segments of 32-wide chunks. A warp walks
-// the (row block, chunk) units of its segment in batches, issuing all of a batch's 16-byte
-// loads before its MMAs. The values feed mma.sync.m16n8k16 (bf16 in, fp32 accumulate)
-// directly as A fragments: the reduction index is permuted inside each 32-wide chunk so
-// that thread (g = lane / 4, t = lane % 4) loads elements 8t .. 8t+7 of rows g and g+8,
-// which become the fragment positions {2t, 2t+1, 2t+8, 2t+9} of two consecutive k16 MMAs;
-// the token operand (8 tokens per MMA) uses the same permutation, so the sum is unchanged.
-// Partial results of the 16 warps meet in shared memory and each output is written once.
+// Compute. The 16 consumer warps form groups of WPS warps (8 for N <= 8, 16 above); group q
+// takes stages q, q + 16/WPS, ..., and its warps split the stage's k-block
+// into 32-wide chunks. Each warp runs mma.sync.m16n8k16 (bf16 in, fp32 accumulate) with the
+// tokens as the A operand (16 rows, rows >= N zero) and the 8 streamed rows as the B
+// operand, one accumulator per chunk so consecutive MMAs do not wait on each other. The
+// reduction index is permuted inside each 32-wide chunk: thread (g = lane / 4, t = lane % 4)
+// reads elements 8t .. 8t+7 of streamed row g and of token rows g, g+8 with one 16-byte load
+// each, which become k-slots {2t, 2t+1, 2t+8, 2t+9} of two consecutive k16 MMAs -- the same
+// permutation on both operands, so the sum is unchanged. Stage rows sit at a pitch of
+// SK * 2 + 16 bytes, so the 8 rows of one fragment load fall in different banks. A warp keeps
+// its token fragments of the current k-block in registers. The WPS partial sums of a stage
+// meet in a shared-memory fp32 accumulator (WPS-way atomic adds); each output is rounded to
+// bf16 and written once.
+//
+// Grid barrier: each CTA adds to a counter whose bit 31 flips when all CTAs have arrived
+// (one CTA adds 2^31 - (G - 1), the others 1; no reset between launches, the counter starts
+// at zero). A CTA reads the bit when it starts -- it cannot flip before that CTA arrives --
+// so arriving is one fire-and-forget release reduction, and waiting is acquire loads.
+//
+// Every wait is bounded: mbarrier waits, the producer's slot waits and the grid barrier give
+// up after the wait limit, record ESPACE_ERR_TIMEOUT and leave; the producer then waits
+// (bounded) for its copies in flight before the CTA exits.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "../../include/espace.h"
 #include "kernels.h"
@@ -30,9 +48,14 @@
 
 namespace espace {
 
-constexpr int DEC_THREADS = 512;
-constexpr int DEC_WARPS = DEC_THREADS / 32;
-constexpr int DEC_MAX_RB = 16;            // 16-row blocks per CTA and phase
+constexpr int DEC_CWARPS = 16;                          // consumer warps
+constexpr int DEC_THREADS = (DEC_CWARPS + 1) * 32;      // + one producer warp
+constexpr int DEC_ROWS = 8;                             // streamed rows per stage
+constexpr int DEC_MAX_STAGES = 12;
+constexpr int DEC_MIN_STAGES = 4;
+constexpr int DEC_SMEM_LIMIT = 232448;                  // opt-in shared memory per block, sm_103
+constexpr int DEC_CONSUMER_BAR = 1;                     // named barrier of the consumer warps
+constexpr int DEC_MAX_GRID = 192;                       // CTAs (one per SM) the cut tables hold
 
 struct DecodeArgs {
     const __nv_bfloat16* A[2];   // streamed matrix of each phase, [R][kdim]
@@ -41,10 +64,41 @@ struct DecodeArgs {
     int R[2], kdim[2], ldo[2];
     int phases;                  // 1 (dense) or 2 (projected)
     int nt;
-    unsigned int* bar;           // grid barrier: [0] arrivals, [1] generation
+    int stages;                  // ring depth
+    int acc_rows;                // rows of the shared accumulator
+    unsigned int* bar;           // grid barrier counter
     int* status;
     uint64_t wait_limit_ns;
+    // CTA b owns rows [cut[p][b], cut[p][b + 1]) of phase p (computed on the host)
+    int cut[2][DEC_MAX_GRID + 1];
 };
+
+// Row cuts: phase 1 split evenly over the G CTAs; phase 2 split so that the bytes of both
+// phases together are balanced (when that keeps the ranges monotone), else evenly. n1, n2:
+// rows; w1, w2: bytes per row (in any common unit). Host code: the kernel reads the tables.
+void decode_cuts(int G, int phases, int n1, int w1, int n2, int w2, int* cut1, int* cut2)
+{
+    for (int b = 0; b <= G; ++b) cut1[b] = static_cast<int>(static_cast<int64_t>(n1) * b / G);
+    if (phases < 2) {
+        for (int b = 0; b <= G; ++b) cut2[b] = 0;
+        return;
+    }
+    const int64_t tot = static_cast<int64_t>(n1) * w1 + static_cast<int64_t>(n2) * w2;
+    const int64_t max1 = (static_cast<int64_t>(n1) + G - 1) / G;
+    if (tot / G >= max1 * w1) {
+        // cumulative phase-2 end after CTA c: the bytes target minus the phase-1 bytes so far;
+        // nondecreasing in c because each CTA's target share covers its phase-1 rows
+        cut2[0] = 0;
+        for (int c = 0; c < G; ++c) {
+            const int64_t t = tot * (c + 1) / G - static_cast<int64_t>(cut1[c + 1]) * w1;
+            const int64_t e = t < 0 ? 0 : t / w2;
+            cut2[c + 1] = static_cast<int>(std::min<int64_t>(e, n2));
+        }
+        cut2[G] = n2;
+    } else {
+        for (int b = 0; b <= G; ++b) cut2[b] = static_cast<int>(static_cast<int64_t>(n2) * b / G);
+    }
+}
 
 __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                                uint32_t a3, uint32_t b0, uint32_t b1)
@@ -56,179 +110,284 @@ __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint3
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Read once: no L1 allocation.
-__device__ __forceinline__ uint4 ldg_stream(const __nv_bfloat16* p)
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar)
 {
-    uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void consumer_sync()
+{
+    asm volatile("bar.sync %0, %1;" ::"n"(DEC_CONSUMER_BAR), "n"(DEC_CWARPS * 32) : "memory");
+}
+
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned* p)
+{
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
 
-__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes)
+// Grid barrier over all CTAs of a cooperative launch, by one thread per CTA; `start` is the
+// counter as this thread read it when the CTA started. Returns false (recording a timeout)
+// if the others did not arrive within the limit.
+__device__ bool grid_arrive_and_wait(unsigned* bar, unsigned start, int* status, uint64_t limit_ns)
 {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+    const unsigned nb = blockIdx.x == 0 ? 0x80000000u - (gridDim.x - 1) : 1u;
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(bar), "r"(nb) : "memory");
+    const uint64_t t0 = globaltimer_ns();
+    uint32_t spins = 0;
+    while (((start ^ ld_acquire_gpu(bar)) & 0x80000000u) == 0) {
+        if ((++spins & 15u) == 0 && globaltimer_ns() - t0 > limit_ns) {
+            atomicExch(status, ESPACE_ERR_TIMEOUT);
+            return false;
+        }
+    }
+    return true;
 }
 
-// Grid-wide barrier for a cooperative launch. Returns false (and records a timeout) if the
-// other CTAs did not arrive within the limit.
-__device__ bool grid_barrier(unsigned int* bar, int* status, uint64_t limit_ns)
+template <int MT, bool HI>
+struct DecodeCfg {
+    static constexpr int SK = 2048;                           // k-block of one stage
+    // consumer warps per stage: each group of WPS warps takes every NG-th stage and splits its
+    // k-block; wider token tiles use larger groups so the fragments fit the register budget
+    static constexpr int WPS = HI ? 16 : 8;
+    static constexpr int NG = DEC_CWARPS / WPS;
+    static constexpr int CPW = SK / 32 / WPS;                 // 32-wide chunks per warp and stage
+    static constexpr int NACC = MT == 2 ? 1 : CPW < 4 ? CPW : 4;   // independent MMA accumulators
+    static constexpr int PITCH = SK * 2 + 16;                 // bytes per stage row
+    static constexpr int STAGE_BYTES = DEC_ROWS * PITCH;
+    // accumulator row pitch (floats): 16 tokens per m16 tile plus 4, so the lanes of one
+    // flush (rows 2t, 2t+1; tokens g) hit 32 different banks
+    static constexpr int NTP = 16 * MT + 4;
+};
+
+// A warp's token fragments for one k-block: v[chunk][m16 tile][row g / row g + 8].
+template <int MT, bool HI>
+struct TokFrag {
+    uint4 v[DecodeCfg<MT, HI>::CPW][MT][HI ? 2 : 1];
+};
+
+// Stage layout. When one k-block covers whole rows (kdim <= SK), a stage's rows are
+// contiguous in HBM and arrive as two runs of 4 rows (two bulk copies), the second 64 bytes
+// past the end of the first, so that the 8 rows of one fragment load still fall in different
+// banks; otherwise each row piece is a copy of its own at a pitch of SK * 2 + 16 bytes.
+template <int PITCH>
+__device__ __forceinline__ int stage_row_offset(int row, int kdim, bool whole)
 {
-    __shared__ int s_ok;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        bool ok = true;
-        volatile unsigned int* gen = bar + 1;
-        const unsigned int my_gen = *gen;
-        __threadfence();
-        const unsigned int arrived = atomicAdd(bar, 1u);
-        if (arrived == gridDim.x - 1) {
-            atomicExch(bar, 0u);
-            __threadfence();
-            atomicAdd(bar + 1, 1u);
-        } else {
-            const uint64_t t0 = globaltimer_ns();
-            while (*gen == my_gen) {
-                if (globaltimer_ns() - t0 > limit_ns) {
-                    atomicExch(status, ESPACE_ERR_TIMEOUT);
-                    ok = false;
-                    break;
+    return whole ? row * kdim * 2 + (row >= 4 ? 64 : 0) : row * PITCH;
+}
+
+template <int MT, bool HI>
+__device__ __forceinline__ void load_tokens(TokFrag<MT, HI>& T, const __nv_bfloat16* B, bool coherent, int kdim,
+                                            int nt, int kb, int u, int g, int t)
+{
+    using C = DecodeCfg<MT, HI>;
+#pragma unroll
+    for (int c = 0; c < C::CPW; ++c) {
+        const int k = kb * C::SK + 32 * (u * C::CPW + c) + 8 * t;
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+            for (int h = 0; h < (HI ? 2 : 1); ++h) {
+                const int n = mt * 16 + g + 8 * h;
+                uint4 v = make_uint4(0, 0, 0, 0);
+                if (n < nt && k < kdim) {
+                    const uint4* p = reinterpret_cast<const uint4*>(B + static_cast<int64_t>(n) * kdim + k);
+                    v = coherent ? __ldcg(p) : __ldg(p);
                 }
-                __nanosleep(64);
+                T.v[c][mt][h] = v;
             }
         }
-        __threadfence();
-        s_ok = ok ? 1 : 0;
     }
-    __syncthreads();
-    return s_ok != 0;
 }
 
-__device__ __forceinline__ void cta_blocks(int R, int& rb0, int& rb1)
+// One stage for the warp with k-part u: the MMAs over its chunks, release of the stage, and
+// the flush of its partial sums into acc (rows r0l .. r0l+rows-1 of the accumulator).
+template <int MT, bool HI>
+__device__ __forceinline__ void consume_stage(const unsigned char* st, uint64_t* empty_bar, const TokFrag<MT, HI>& T,
+                                              int ksz, bool whole, int rows, int r0l, int nt, float* acc, int u,
+                                              int lane)
 {
-    const int blocks = (R + 15) / 16;
-    rb0 = static_cast<int>(static_cast<int64_t>(blocks) * blockIdx.x / gridDim.x);
-    rb1 = static_cast<int>(static_cast<int64_t>(blocks) * (blockIdx.x + 1) / gridDim.x);
-}
-
-// L2 prefetch of this CTA's rows of A (contiguous), 64 KB per request.
-__device__ __forceinline__ void prefetch_rows(const __nv_bfloat16* A, int R, int kdim)
-{
-    int rb0, rb1;
-    cta_blocks(R, rb0, rb1);
-    const int r_end = min(rb1 * 16, R);
-    if (r_end <= rb0 * 16) return;
-    const char* base = reinterpret_cast<const char*>(A + static_cast<int64_t>(rb0) * 16 * kdim);
-    const int64_t bytes = static_cast<int64_t>(r_end - rb0 * 16) * kdim * 2;
-    for (int64_t off = 0; off < bytes; off += 65536)
-        prefetch_l2_bulk(base + off, static_cast<uint32_t>(bytes - off < 65536 ? bytes - off : 65536));
-}
-
-// One phase: out[n][r] = bf16(sum_k B[n][k] A[r][k]) for this CTA's row blocks. Tokens
-// n < nt of B are read through the cache (`b_coherent`: through L2 only, for data written
-// earlier in the same launch). acc_s: zeroed [DEC_MAX_RB * 16][NTP] fp32.
-template <int NTILES, int BATCH>
-__device__ void decode_phase(const __nv_bfloat16* __restrict__ A, const __nv_bfloat16* B, bool b_coherent,
-                             int R, int kdim, int nt, float* acc_s, __nv_bfloat16* __restrict__ out, int ldo)
-{
-    constexpr int NTP = 8 * NTILES;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    using C = DecodeCfg<MT, HI>;
     const int g = lane >> 2, t = lane & 3;
-    int rb0, rb1;
-    cta_blocks(R, rb0, rb1);
-    const int chunks = (kdim + 31) / 32;
-    const int per_warp = (chunks + DEC_WARPS - 1) / DEC_WARPS;
-    const int c_begin = min(warp * per_warp, chunks);
-    const int nch = min(c_begin + per_warp, chunks) - c_begin;     // chunks of this warp
-    const int units = (rb1 - rb0) * nch;
-
-    // token rows this thread feeds into the B fragments (rows past nt read as zero)
-    const __nv_bfloat16* brow[NTILES];
-    bool bvalid[NTILES];
+    st += stage_row_offset<C::PITCH>(g, ksz, whole);
+    float d[C::NACC][MT][4];
 #pragma unroll
-    for (int j = 0; j < NTILES; ++j) {
-        const int n = j * 8 + g;
-        bvalid[j] = n < nt;
-        brow[j] = B + static_cast<int64_t>(bvalid[j] ? n : 0) * kdim;
-    }
-
-    float c[NTILES][4];
+    for (int q = 0; q < C::NACC; ++q)
 #pragma unroll
-    for (int j = 0; j < NTILES; ++j) c[j][0] = c[j][1] = c[j][2] = c[j][3] = 0.f;
-
-    for (int u0 = 0; u0 < units; u0 += BATCH) {
-        // every load of the batch (A rows and token rows) is issued before the first MMA
-        uint4 lo[BATCH], hi[BATCH], bf[BATCH][NTILES];
+        for (int mt = 0; mt < MT; ++mt) d[q][mt][0] = d[q][mt][1] = d[q][mt][2] = d[q][mt][3] = 0.f;
 #pragma unroll
-        for (int i = 0; i < BATCH; ++i) {
-            const int u = u0 + i;
-            lo[i] = hi[i] = make_uint4(0, 0, 0, 0);
+    for (int c = 0; c < C::CPW; ++c) {
+        const int kl = 32 * (u * C::CPW + c) + 8 * t;
+        uint4 w = make_uint4(0, 0, 0, 0);
+        if (kl < ksz) w = *reinterpret_cast<const uint4*>(st + kl * 2);
 #pragma unroll
-            for (int j = 0; j < NTILES; ++j) bf[i][j] = make_uint4(0, 0, 0, 0);
-            if (u < units) {
-                const int rb = rb0 + u / nch;
-                const int k = (c_begin + u % nch) * 32 + 8 * t;
-                const int r_lo = rb * 16 + g, r_hi = r_lo + 8;
-                if (k < kdim) {
-                    if (r_lo < R) lo[i] = ldg_stream(A + static_cast<int64_t>(r_lo) * kdim + k);
-                    if (r_hi < R) hi[i] = ldg_stream(A + static_cast<int64_t>(r_hi) * kdim + k);
-#pragma unroll
-                    for (int j = 0; j < NTILES; ++j)
-                        if (bvalid[j])
-                            bf[i][j] = b_coherent ? __ldcg(reinterpret_cast<const uint4*>(brow[j] + k))
-                                                  : __ldg(reinterpret_cast<const uint4*>(brow[j] + k));
-                }
-            }
-        }
-#pragma unroll
-        for (int i = 0; i < BATCH; ++i) {
-            const int u = u0 + i;
-            if (u >= units) break;                       // uniform across the warp
-#pragma unroll
-            for (int j = 0; j < NTILES; ++j) {
-                mma_bf16_16816(c[j], lo[i].x, hi[i].x, lo[i].y, hi[i].y, bf[i][j].x, bf[i][j].y);
-                mma_bf16_16816(c[j], lo[i].z, hi[i].z, lo[i].w, hi[i].w, bf[i][j].z, bf[i][j].w);
-            }
-            if ((u + 1) % nch == 0) {                    // last chunk of this row block
-                float* slot = acc_s + (u / nch) * 16 * NTP;
-#pragma unroll
-                for (int j = 0; j < NTILES; ++j) {
-                    atomicAdd(slot + g * NTP + 8 * j + 2 * t, c[j][0]);
-                    atomicAdd(slot + g * NTP + 8 * j + 2 * t + 1, c[j][1]);
-                    atomicAdd(slot + (g + 8) * NTP + 8 * j + 2 * t, c[j][2]);
-                    atomicAdd(slot + (g + 8) * NTP + 8 * j + 2 * t + 1, c[j][3]);
-                    c[j][0] = c[j][1] = c[j][2] = c[j][3] = 0.f;
-                }
-            }
+        for (int mt = 0; mt < MT; ++mt) {
+            const uint4 lo = T.v[c][mt][0];
+            const uint4 hi = HI ? T.v[c][mt][HI ? 1 : 0] : make_uint4(0, 0, 0, 0);
+            mma_bf16_16816(d[c % C::NACC][mt], lo.x, hi.x, lo.y, hi.y, w.x, w.y);
+            mma_bf16_16816(d[c % C::NACC][mt], lo.z, hi.z, lo.w, hi.w, w.z, w.w);
         }
     }
-    __syncthreads();
-    const int rows = (rb1 - rb0) * 16;
-    for (int i = threadIdx.x; i < rows * NTP; i += blockDim.x) {
-        const int n = i / rows, rr = i - n * rows;           // token-major: coalesced stores
-        const int r = rb0 * 16 + rr;
-        if (n < nt && r < R) out[static_cast<int64_t>(n) * ldo + r] = __float2bfloat16_rn(acc_s[rr * NTP + n]);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty_bar);
+#pragma unroll
+    for (int q = 1; q < C::NACC; ++q)
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) d[0][mt][e] += d[q][mt][e];
+    // d[0][mt]: {token g, rows 2t, 2t+1}, {token g+8, rows 2t, 2t+1}; rows past the CTA's range
+    // were not copied and are not flushed
+    const bool r_lo = 2 * t < rows, r_hi = 2 * t + 1 < rows;
+    float* a = acc + (r0l + 2 * t) * C::NTP;
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+        const int n = mt * 16 + g;
+        if (n < nt) {
+            if (r_lo) atomicAdd(a + n, d[0][mt][0]);
+            if (r_hi) atomicAdd(a + C::NTP + n, d[0][mt][1]);
+        }
+        if (HI && n + 8 < nt) {
+            if (r_lo) atomicAdd(a + n + 8, d[0][mt][2]);
+            if (r_hi) atomicAdd(a + C::NTP + n + 8, d[0][mt][3]);
+        }
     }
-    __syncthreads();
-    for (int i = threadIdx.x; i < rows * NTP; i += blockDim.x) acc_s[i] = 0.f;
-    __syncthreads();
 }
 
-template <int NTILES>
+template <int MT, bool HI>
 __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs a)
 {
-    constexpr int NTP = 8 * NTILES;
-    constexpr int BATCH = NTILES == 1 ? 8 : NTILES == 2 ? 4 : 2;
-    __shared__ float acc_s[DEC_MAX_RB * 16 * NTP];
-    // rows of the second matrix towards L2 while the first one streams
-    if (threadIdx.x == 0 && a.phases > 1) prefetch_rows(a.A[1], a.R[1], a.kdim[1]);
-    for (int i = threadIdx.x; i < DEC_MAX_RB * 16 * NTP; i += blockDim.x) acc_s[i] = 0.f;
+    using C = DecodeCfg<MT, HI>;
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ __align__(8) uint64_t full[DEC_MAX_STAGES];
+    __shared__ __align__(8) uint64_t empty[DEC_MAX_STAGES];
+    __shared__ int abort_s;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int rb0[2] = {a.cut[0][blockIdx.x], a.cut[1][blockIdx.x]};   // rows [rb0[p], rb1[p])
+    const int rb1[2] = {a.cut[0][blockIdx.x + 1], a.cut[1][blockIdx.x + 1]};
+
+
+    float* acc = reinterpret_cast<float*>(smem);
+    unsigned char* ring = smem + ((static_cast<size_t>(a.acc_rows) * C::NTP * 4 + 127) & ~static_cast<size_t>(127));
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < a.stages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], C::WPS);
+        }
+        abort_s = 0;
+        fence_barrier_init();
+    }
+    for (int i = threadIdx.x; i < a.acc_rows * C::NTP; i += blockDim.x) acc[i] = 0.f;
     __syncthreads();
-    decode_phase<NTILES, BATCH>(a.A[0], a.B[0], false, a.R[0], a.kdim[0], a.nt, acc_s, a.out[0], a.ldo[0]);
-    if (a.phases > 1) {
-        if (!grid_barrier(a.bar, a.status, a.wait_limit_ns)) return;
-        decode_phase<NTILES, BATCH>(a.A[1], a.B[1], true, a.R[1], a.kdim[1], a.nt, acc_s, a.out[1], a.ldo[1]);
+    volatile int* abort = &abort_s;
+
+    if (warp == DEC_CWARPS) {
+        // ------------------------------------------------------------ producer (one thread)
+        if (lane != 0) return;
+        int j = 0;
+#pragma unroll
+        for (int p = 0; p < 2; ++p) {
+            if (p >= a.phases || *abort) break;
+            const __nv_bfloat16* A = a.A[p];
+            const int kdim = a.kdim[p];
+            const int nkb = (kdim + C::SK - 1) / C::SK;
+            for (int kb = 0; kb < nkb && !*abort; ++kb) {
+                const int ksz = min(C::SK, kdim - kb * C::SK);
+                for (int r = rb0[p]; r < rb1[p]; r += DEC_ROWS, ++j) {
+                    const int slot = j % a.stages;
+                    if (j >= a.stages &&
+                        !mbar_wait(&empty[slot], static_cast<uint32_t>(j / a.stages - 1) & 1u, abort, a.status,
+                                   a.wait_limit_ns, ESPACE_ERR_TIMEOUT))
+                        break;
+                    const int rows = min(DEC_ROWS, rb1[p] - r);
+                    mbar_arrive_expect_tx(&full[slot], static_cast<uint32_t>(rows * ksz * 2));
+                    unsigned char* dst = ring + static_cast<size_t>(slot) * C::STAGE_BYTES;
+                    const __nv_bfloat16* src = A + static_cast<int64_t>(r) * kdim + kb * C::SK;
+                    if (kdim <= C::SK) {
+                        // whole rows: two runs of up to 4 contiguous rows
+                        const int lo = min(rows, 4);
+                        bulk_load(dst, src, static_cast<uint32_t>(lo * kdim * 2), &full[slot]);
+                        if (rows > 4)
+                            bulk_load(dst + stage_row_offset<C::PITCH>(4, kdim, true), src + static_cast<int64_t>(4) * kdim,
+                                      static_cast<uint32_t>((rows - 4) * kdim * 2), &full[slot]);
+                    } else {
+                        for (int q = 0; q < rows; ++q)
+                            bulk_load(dst + q * C::PITCH, src + static_cast<int64_t>(q) * kdim,
+                                      static_cast<uint32_t>(ksz * 2), &full[slot]);
+                    }
+                }
+            }
+        }
+        if (*abort) {
+            // let the copies already issued land before the CTA's shared memory goes away
+            volatile int never = 0;
+            for (int q = max(0, j - a.stages); q < j; ++q)
+                mbar_wait(&full[q % a.stages], static_cast<uint32_t>(q / a.stages) & 1u, &never, a.status,
+                          a.wait_limit_ns, ESPACE_ERR_TIMEOUT);
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------------- consumers (16 warps)
+    const int group = warp / C::WPS, u = warp % C::WPS;
+    // the grid barrier's bit before this CTA arrives (it cannot flip earlier)
+    const unsigned bar_start = (a.phases > 1 && threadIdx.x == 0) ? ld_acquire_gpu(a.bar) : 0u;
+    int j0 = 0;   // ring index of the phase's first stage
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+        if (p >= a.phases) break;
+        const __nv_bfloat16* B = a.B[p];
+        const bool coherent = p > 0;   // Z was written earlier in this launch
+        const int kdim = a.kdim[p];
+        const int nkb = (kdim + C::SK - 1) / C::SK;
+        const int nrs = (rb1[p] - rb0[p] + DEC_ROWS - 1) / DEC_ROWS;   // row stages per k-block
+        // stages run k-block-major; this group takes stages group, group + NG, ...
+        TokFrag<MT, HI> T;
+        int cur_kb = -1;
+        for (int i = group; i < nkb * nrs; i += C::NG) {
+            const int kb = i / nrs, rs = i - kb * nrs;
+            if (kb != cur_kb) {
+                load_tokens<MT, HI>(T, B, coherent, kdim, a.nt, kb, u, lane >> 2, lane & 3);
+                cur_kb = kb;
+            }
+            const int j = j0 + i;
+            const int slot = j % a.stages;
+            if (*abort) continue;
+            if (!mbar_wait(&full[slot], static_cast<uint32_t>(j / a.stages) & 1u, abort, a.status, a.wait_limit_ns,
+                           ESPACE_ERR_TIMEOUT))
+                continue;
+            const int r0l = rs * DEC_ROWS;
+            consume_stage<MT, HI>(ring + static_cast<size_t>(slot) * C::STAGE_BYTES, &empty[slot], T,
+                                  min(C::SK, kdim - kb * C::SK), kdim <= C::SK, min(DEC_ROWS, rb1[p] - rb0[p] - r0l),
+                                  r0l, a.nt, acc, u, lane);
+        }
+        j0 += nkb * nrs;
+        consumer_sync();
+        // outputs of this CTA's rows, token-major (coalesced); then clear the accumulator
+        const int rows = rb1[p] - rb0[p];
+        if (!*abort) {
+            for (int i = threadIdx.x; i < rows * a.nt; i += DEC_CWARPS * 32) {
+                const int n = i / rows, rr = i - n * rows;
+                a.out[p][static_cast<int64_t>(n) * a.ldo[p] + rb0[p] + rr] = __float2bfloat16_rn(acc[rr * C::NTP + n]);
+            }
+        }
+        consumer_sync();
+        for (int i = threadIdx.x; i < rows * C::NTP; i += DEC_CWARPS * 32) acc[i] = 0.f;
+        if (p + 1 < a.phases) {
+            // every Z of this CTA is stored (consumer_sync above); wait for all CTAs
+            if (threadIdx.x == 0) {
+                const bool ok = !*abort && grid_arrive_and_wait(a.bar, bar_start, a.status, a.wait_limit_ns);
+                if (!ok) *abort = 1;
+            }
+        }
+        consumer_sync();
     }
 }
 
@@ -236,46 +395,120 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
 
 namespace {
 
-int ntiles_for(int nt) { return nt <= 8 ? 1 : nt <= 16 ? 2 : 4; }
+struct DecodePlan {
+    int mt = 1;
+    bool hi = false;
+    int stages = 0;
+    int acc_rows = 0;
+    int smem = 0;
+    int cut[2][DEC_MAX_GRID + 1] = {};
+};
 
-template <int NTILES>
-cudaError_t launch(DecodeArgs& a, const DeviceInfo* dev, cudaStream_t stream)
+int ntp_of(int mt) { return 16 * mt + 4; }
+int stage_bytes_of(int) { return DecodeCfg<1, false>::STAGE_BYTES; }
+
+bool compute_plan(int mt, int phases, int R0, int k0, int R1, int k1, int G, DecodePlan* pl)
 {
-    auto kern = decode_kernel<NTILES>;
+    pl->mt = mt;
+    decode_cuts(G, phases, R0, k0, phases > 1 ? R1 : 0, phases > 1 ? k1 : 1, pl->cut[0], pl->cut[1]);
+    int max_rows = 1;
+    for (int b = 0; b < G; ++b)
+        max_rows = std::max(max_rows, std::max(pl->cut[0][b + 1] - pl->cut[0][b], pl->cut[1][b + 1] - pl->cut[1][b]));
+    max_rows = (max_rows + DEC_ROWS - 1) / DEC_ROWS * DEC_ROWS;
+    if (static_cast<int64_t>(max_rows) * ntp_of(mt) * 4 > DEC_SMEM_LIMIT) return false;
+    pl->acc_rows = max_rows;
+    const int acc_bytes = (pl->acc_rows * ntp_of(mt) * 4 + 127) & ~127;
+    const int sb = stage_bytes_of(mt);
+    pl->stages = std::min(DEC_MAX_STAGES, (DEC_SMEM_LIMIT - 1024 - acc_bytes) / sb);
+    if (pl->stages < DEC_MIN_STAGES) return false;
+    pl->smem = acc_bytes + pl->stages * sb;
+    return true;
+}
+
+// Plans are cached by shape: a decode step repeats the same few layer shapes.
+bool make_plan(int nt, int phases, int R0, int k0, int R1, int k1, int G, DecodePlan* plan)
+{
+    if (nt < 1 || nt > DECODE_MAX_TOKENS || G < 1 || G > DEC_MAX_GRID) return false;
+    if (k0 < 8 || k0 % 8 != 0 || R0 < 1) return false;
+    if (phases > 1 && (k1 < 8 || k1 % 8 != 0 || R1 < 1)) return false;
+    if (phases < 2) R1 = k1 = 0;
+    const int mt = nt <= 16 ? 1 : 2;
+    struct Entry {
+        bool valid = false, ok = false;
+        int key[7] = {};
+        DecodePlan plan;
+    };
+    static Entry cache[16];
+    static int next = 0;
+    static std::mutex mu;
+    const int key[7] = {mt, phases, R0, k0, R1, k1, G};
+    std::lock_guard<std::mutex> lock(mu);
+    for (Entry& e : cache)
+        if (e.valid && std::equal(key, key + 7, e.key)) {
+            if (!e.ok) return false;
+            *plan = e.plan;
+            plan->hi = nt > 8;
+            return true;
+        }
+    Entry& e = cache[next];
+    next = (next + 1) % 16;
+    e.valid = true;
+    std::copy(key, key + 7, e.key);
+    e.ok = compute_plan(mt, phases, R0, k0, R1, k1, G, &e.plan);
+    if (!e.ok) return false;
+    *plan = e.plan;
+    plan->hi = nt > 8;
+    return true;
+}
+
+template <int MT, bool HI>
+cudaError_t launch_t(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev, cudaStream_t stream)
+{
+    auto kern = decode_kernel<MT, HI>;
     static bool configured[64] = {};
     if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
     if (!configured[dev->device]) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             DEC_SMEM_LIMIT - 1024);
+        if (e != cudaSuccess) return e;
         int per_sm = 0;
-        cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, DEC_THREADS, 0);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, DEC_THREADS, DEC_SMEM_LIMIT - 1024);
         if (e != cudaSuccess) return e;
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
         configured[dev->device] = true;
     }
+    a.stages = pl.stages;
+    a.acc_rows = pl.acc_rows;
+    std::copy(&pl.cut[0][0], &pl.cut[0][0] + 2 * (DEC_MAX_GRID + 1), &a.cut[0][0]);
     if (a.phases == 1) {
         // no grid barrier: an ordinary launch
-        kern<<<dev->num_sms, DEC_THREADS, 0, stream>>>(a);
+        kern<<<dev->num_sms, DEC_THREADS, pl.smem, stream>>>(a);
         return cudaGetLastError();
     }
     void* params[] = {&a};
     return cudaLaunchCooperativeKernel(reinterpret_cast<void*>(kern), dim3(dev->num_sms), dim3(DEC_THREADS),
-                                       params, 0, stream);
+                                       params, static_cast<size_t>(pl.smem), stream);
 }
 
-cudaError_t launch_any(DecodeArgs& a, const DeviceInfo* dev, cudaStream_t stream)
+cudaError_t launch_any(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev, cudaStream_t stream)
 {
-    const int nti = ntiles_for(a.nt);
-    if (nti == 1) return launch<1>(a, dev, stream);
-    if (nti == 2) return launch<2>(a, dev, stream);
-    return launch<4>(a, dev, stream);
+    if (pl.mt == 2) return launch_t<2, true>(a, pl, dev, stream);
+    if (pl.hi) return launch_t<1, true>(a, pl, dev, stream);
+    return launch_t<1, false>(a, pl, dev, stream);
 }
 
 }  // namespace
 
 bool decode_supported(int nt, int K, int Lp, int M, int num_sms)
 {
-    if (nt < 1 || nt > DECODE_MAX_TOKENS || K % 8 != 0 || Lp % 8 != 0 || num_sms < 1) return false;
-    const int blocks = std::max((Lp + 15) / 16, (M + 15) / 16);
-    return (blocks + num_sms - 1) / num_sms <= DEC_MAX_RB;
+    DecodePlan pl;
+    return make_plan(nt, 2, Lp, K, M, Lp, num_sms, &pl);
+}
+
+bool decode_dense_supported(int nt, int K, int M, int num_sms)
+{
+    DecodePlan pl;
+    return make_plan(nt, 1, M, K, 0, 0, num_sms, &pl);
 }
 
 cudaError_t launch_decode_forward(const void* PT, const void* WfT, const void* X, void* Z, void* Y,
@@ -284,7 +517,8 @@ cudaError_t launch_decode_forward(const void* PT, const void* WfT, const void* X
 {
     DeviceInfo* dev = nullptr;
     if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
-    if (!decode_supported(nt, K, Lp, M, dev->num_sms)) return cudaErrorInvalidValue;
+    DecodePlan pl;
+    if (!make_plan(nt, 2, Lp, K, M, Lp, dev->num_sms, &pl)) return cudaErrorInvalidValue;
     DecodeArgs a{};
     a.A[0] = static_cast<const __nv_bfloat16*>(PT);
     a.B[0] = static_cast<const __nv_bfloat16*>(X);
@@ -303,7 +537,7 @@ cudaError_t launch_decode_forward(const void* PT, const void* WfT, const void* X
     a.bar = grid_bar;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
-    return launch_any(a, dev, stream);
+    return launch_any(a, pl, dev, stream);
 }
 
 cudaError_t launch_decode_dense(const void* W, const void* X, void* Y, int K, int M, int nt,
@@ -311,7 +545,8 @@ cudaError_t launch_decode_dense(const void* W, const void* X, void* Y, int K, in
 {
     DeviceInfo* dev = nullptr;
     if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
-    if (!decode_supported(nt, K, 8, M, dev->num_sms)) return cudaErrorInvalidValue;
+    DecodePlan pl;
+    if (!make_plan(nt, 1, M, K, 0, 0, dev->num_sms, &pl)) return cudaErrorInvalidValue;
     DecodeArgs a{};
     a.A[0] = static_cast<const __nv_bfloat16*>(W);
     a.B[0] = static_cast<const __nv_bfloat16*>(X);
@@ -324,7 +559,7 @@ cudaError_t launch_decode_dense(const void* W, const void* X, void* Y, int K, in
     a.bar = nullptr;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
-    return launch_any(a, dev, stream);
+    return launch_any(a, pl, dev, stream);
 }
 
 }  // namespace espace

@@ -169,7 +169,7 @@ struct espace_proj_s {
     std::vector<double> evals;     // K eigenvalues, decreasing (if calibrated)
     uint16_t* Z = nullptr;         // [zcap][Lp] bf16 scratch for the rank-L intermediate
     int64_t zcap = 0;
-    unsigned int* bar = nullptr;   // grid barrier of the decode kernel (2 words, zeroed)
+    unsigned int* bar = nullptr;   // grid barrier counter of the decode kernel (zeroed)
     int* ready = nullptr;          // fused forward: 2 x ceil(zcap / 256) zeroed counters
     std::mutex mu;                 // guards Z growth
 };
@@ -664,7 +664,7 @@ int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_
     int rc = device_info(&dev);
     if (rc != ESPACE_OK) return rc;
     // few tokens: stream W once through the decode kernel; otherwise the tcgen05 GEMM
-    if (N <= DECODE_MAX_TOKENS && decode_supported(static_cast<int>(N), static_cast<int>(K), 8, static_cast<int>(M), dev->num_sms)) {
+    if (N <= DECODE_MAX_TOKENS && decode_dense_supported(static_cast<int>(N), static_cast<int>(K), static_cast<int>(M), dev->num_sms)) {
         CUDA_TRY(launch_decode_dense(W_dev, X_dev, Y_dev, static_cast<int>(K), static_cast<int>(M), static_cast<int>(N),
                                      static_cast<cudaStream_t>(stream)),
                  "espace_dense_forward: decode launch");

@@ -42,8 +42,9 @@ constexpr int DECODE_MAX_TOKENS = 32;
 
 // Decode-shaped forward (nt <= DECODE_MAX_TOKENS) in one cooperative launch: Z[nt][Lp] = X P
 // from P^T [Lp][K], a grid barrier, then Y[nt][M] = Z W' from W'^T [M][Lp]; each matrix
-// streamed from HBM once. grid_bar: two zeroed unsigned ints owned by the caller (one launch
-// at a time may use them).
+// streamed from HBM once. grid_bar: one unsigned int owned by the caller, zero before the
+// first launch and left at a multiple of 2^31 by every launch that completes (one launch at a
+// time may use it).
 cudaError_t launch_decode_forward(const void* PT, const void* WfT, const void* X, void* Z, void* Y,
                                   int K, int Lp, int M, int nt, unsigned int* grid_bar,
                                   cudaStream_t stream);
@@ -51,6 +52,7 @@ cudaError_t launch_decode_forward(const void* PT, const void* WfT, const void* X
 cudaError_t launch_decode_dense(const void* W, const void* X, void* Y, int K, int M, int nt,
                                 cudaStream_t stream);
 bool decode_supported(int nt, int K, int Lp, int M, int num_sms);
+bool decode_dense_supported(int nt, int K, int M, int num_sms);
 
 // Xn[t][k] = bf16(X[t][k] / ||x_t||) (0 for a zero token), fp32 norms.
 cudaError_t launch_normalize_rows(const void* X, int64_t N, int K, void* Xn, cudaStream_t stream);
