@@ -427,7 +427,8 @@ def graph_time_us(call, per_graph=20, replays=10):
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(side):
-        for i in range(3):
+        # every call of the graph once: scratch and workspaces grow outside the capture
+        for i in range(per_graph):
             call(i)
     torch.cuda.current_stream().wait_stream(side)
     torch.cuda.synchronize()

@@ -146,17 +146,21 @@ void espace_proj_destroy(espace_proj_t p);
 
 /* Async. Y = (P^T W)^T (P^T X) for the N tokens of X_dev ([N][K] bf16) into Y_dev
  * ([N][M] bf16): Z = X P is accumulated in fp32 and rounded to bf16 (the paper computes in
- * BF16, Sec. A.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. Small N runs
- * a bandwidth-bound kernel that streams P and W' once; larger N runs the tcgen05
- * tensor-core path. N = 0 is a no-op. The first call with a larger N than any before on
- * this handle allocates the Z scratch (synchronously); later calls allocate nothing. */
+ * BF16, Sec. A.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 32 runs
+ * a bandwidth-bound kernel that streams P and W' once; N <= 256 runs two tcgen05 launches
+ * with the weights as the 128-row operand (phase 1 splits its reduction over the SMs and
+ * adds the fp32 partials in a fixed order, so results are reproducible bit for bit);
+ * larger N runs one persistent tcgen05 launch holding both products. N = 0 is a no-op.
+ * The first call with a larger N than any before on this handle allocates the Z scratch
+ * and, for N <= 256, the split workspace (synchronously); later calls allocate nothing. */
 int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev,
                           void* stream);
 
 /* As espace_linear_forward with the kernel family chosen by the caller:
  *   0 automatic;
- *   1 tcgen05 tensor-core kernels: one persistent launch holding both products when N, L
- *     and M exceed 128 (Z stays in L2 between them), else one launch per product;
+ *   1 tcgen05 tensor-core kernels: for N <= 256 one launch per product with the weights as
+ *     the 128-row operand; above, one persistent launch holding both products when L and M
+ *     exceed 128 (Z stays in L2 between them), else one launch per product;
  *   2 the decode-shaped streaming kernel (ESPACE_ERR_SHAPE if N > 32 or the layer is too
  *     large for it);
  *   3 tcgen05 kernels, always one launch per product (Z through the scratch buffer). */
@@ -194,8 +198,10 @@ int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev, int64_t N,
                                   void* stream);
 
 /* Async. The uncompressed layer of Eq. 1, Y = W^T X, as Y_dev[N][M] = X_dev[N][K] W_dev^T
- * with W_dev in [M][K] layout, on the same tcgen05 kernel with fp32 accumulation and bf16
- * output: the baseline the projected layer is measured against. */
+ * with W_dev in [M][K] layout, with fp32 accumulation and bf16 output on the same kernel
+ * families as the projected layer (N <= 32: the streaming kernel; N <= 256: tcgen05 with
+ * the weights as the 128-row operand, no split; above: tcgen05): the baseline the
+ * projected layer is measured against. */
 int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev,
                          int64_t M, void* Y_dev, void* stream);
 

@@ -171,7 +171,9 @@ struct espace_proj_s {
     int64_t zcap = 0;
     unsigned int* bar = nullptr;   // grid barrier counter of the decode kernel (zeroed)
     int* ready = nullptr;          // fused forward: 2 x ceil(zcap / 256) zeroed counters
-    std::mutex mu;                 // guards Z growth
+    float* part = nullptr;         // split reductions of the few-token products (fp32)
+    int64_t part_cap = 0;
+    std::mutex mu;                 // guards scratch growth
 };
 
 extern "C" {
@@ -549,6 +551,7 @@ void espace_proj_destroy(espace_proj_t p)
     if (p->Z) cudaFree(p->Z);
     if (p->bar) cudaFree(p->bar);
     if (p->ready) cudaFree(p->ready);
+    if (p->part) cudaFree(p->part);
     delete p;
 }
 
@@ -580,6 +583,29 @@ static int ensure_z(espace_proj_s* p, int64_t N, cudaStream_t st)
     p->zcap = cap;
     return ESPACE_OK;
 }
+
+// Workspace of the swapped products (phase 1: P^T against X; phase 2: W'^T against Z) for
+// n tokens, grown when a plan needs more.
+static int ensure_swap(espace_proj_s* p, int n, int num_sms, cudaStream_t st)
+{
+    const SwapPlan a = gemm_swap_plan(static_cast<int>(p->Lp), n, static_cast<int>(p->K), num_sms, true);
+    const SwapPlan b = gemm_swap_plan(static_cast<int>(p->M), n, static_cast<int>(p->Lp), num_sms, true);
+    const int64_t part = std::max(a.part_elems, b.part_elems);
+    std::lock_guard<std::mutex> lock(p->mu);
+    if (part == 0 || p->part_cap >= part) return ESPACE_OK;
+    CUDA_TRY(cudaStreamSynchronize(st), "forward: sync before workspace growth");
+    if (p->part) cudaFree(p->part);
+    p->part = nullptr;
+    p->part_cap = 0;
+    cudaError_t e = cudaMalloc(&p->part, sizeof(float) * part);
+    if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "forward: split workspace: %s", cudaGetErrorString(e));
+    p->part_cap = part;
+    return ESPACE_OK;
+}
+
+// Tokens served by the swapped tcgen05 products (between the decode kernel and the fused
+// CTA-pair launch).
+static bool swap_forward_applies(int n, int path) { return n <= SWAP_MAX_TOKENS && path != ESPACE_PATH_TENSOR_SPLIT; }
 
 int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev, void* stream,
                                int path)
@@ -614,6 +640,13 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
         CUDA_TRY(launch_decode_forward(p->PT, p->WfT, X_dev, p->Z, Y_dev, K, Lp, M, n, p->bar, st),
                  "forward: decode kernel");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+    } else if (swap_forward_applies(n, path)) {
+        // few tokens: the weights are the 128-row operand; phase 1 splits its reduction
+        rc = ensure_swap(p, n, dev->num_sms, st);
+        if (rc != ESPACE_OK) return rc;
+        CUDA_TRY(launch_gemm_swap(p->PT, K, X_dev, K, Lp, n, K, p->Z, Lp, p->part, st), "forward: phase 1");
+        if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+        CUDA_TRY(launch_gemm_swap(p->WfT, Lp, p->Z, Lp, M, n, Lp, Y_dev, M, p->part, st), "forward: phase 2");
     } else if (path != ESPACE_PATH_TENSOR_SPLIT && fused_forward_applies(n, Lp, M)) {
         // one persistent launch holds both products; the phase event marks its start
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
@@ -641,6 +674,12 @@ int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path)
               Lp = static_cast<int>(p->Lp);
     const bool small_ok = N <= DECODE_MAX_TOKENS && decode_supported(n, K, Lp, M, dev->num_sms);
     if (path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok)) return small_ok ? 1 : -1;
+    if (swap_forward_applies(n, path)) {
+        // one launch per product, plus one per split reduction
+        const int a = gemm_swap_plan(Lp, n, K, dev->num_sms, true).ksplit > 1 ? 2 : 1;
+        const int b = gemm_swap_plan(M, n, Lp, dev->num_sms, true).ksplit > 1 ? 2 : 1;
+        return a + b;
+    }
     if (path != ESPACE_PATH_TENSOR_SPLIT && fused_forward_applies(n, Lp, M)) return 1;
     return 2;
 }
@@ -668,6 +707,13 @@ int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_
         CUDA_TRY(launch_decode_dense(W_dev, X_dev, Y_dev, static_cast<int>(K), static_cast<int>(M), static_cast<int>(N),
                                      static_cast<cudaStream_t>(stream)),
                  "espace_dense_forward: decode launch");
+        return ESPACE_OK;
+    }
+    if (N <= SWAP_MAX_TOKENS) {
+        // few tokens: the weight rows span the grid (no split: no workspace without a handle)
+        CUDA_TRY(launch_gemm_swap(W_dev, K, X_dev, K, static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), Y_dev,
+                                  M, nullptr, static_cast<cudaStream_t>(stream)),
+                 "espace_dense_forward: launch");
         return ESPACE_OK;
     }
     CUDA_TRY(launch_gemm_tn(X_dev, K, W_dev, K, static_cast<int>(N), static_cast<int>(M), static_cast<int>(K), Y_dev, M,

@@ -31,6 +31,20 @@ cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ld
 cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,
                                  int K, int Lp, int M, int* ready, int* done, cudaStream_t stream);
 
+// Swapped product for few tokens (ntok <= 256): out[n][r] (bf16, leading dimension ldo) =
+// sum_k W[r][k] X[n][k], the weights as the 128-row tcgen05 operand, the tile stored
+// transposed. The reduction splits over CTAs (ksplit > 1) only when a workspace `part` of
+// the plan's part_elems fp32 values (made with allow_split) is given; a second launch then
+// adds the partials in split order.
+struct SwapPlan {
+    int bn = 128, tiles = 0, kblocks = 0, ksplit = 1, kb_per_split = 0;
+    int64_t ld_part = 0, part_elems = 0;
+};
+SwapPlan gemm_swap_plan(int rows, int ntok, int kdim, int num_sms, bool allow_split);
+cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t ldx, int rows, int ntok, int kdim,
+                             void* out, int64_t ldo, float* part, cudaStream_t stream);
+constexpr int SWAP_MAX_TOKENS = 256;
+
 // Whether the CTA-pair kernels are enabled (ESPACE_DISABLE_PAIR_GEMM=1 turns them off).
 bool pair_kernel_enabled();
 

@@ -9,7 +9,11 @@
 // Two operand layouts share the kernel:
 //   * K-major ("TN"): C[r][c] = sum_k A[r][k] B[c][k] -- the projected layer's two products
 //     Z = X P and Y = Z W' (with P^T and W'^T stored row-major), the fold W'^T = W P and
-//     the dense baseline Y = X W^T;
+//     the dense baseline Y = X W^T. For few tokens the operands swap (A = the weights, 128
+//     rows per tile; B = the tokens) and the epilogue stores the tile transposed, so that
+//     the grid spans the weight rows; a reduction split over CTAs writes fp32 partial tiles
+//     to a workspace, and a second launch adds them in split order (deterministic) and
+//     stores the bf16 result;
 //   * M/N-major: S[i][j] += sum_t X[t][i] X[t][j] -- the autocorrelation of Eq. 4, read
 //     straight from token-major X, upper-triangle tiles only, split over tokens with fp32
 //     atomics.
@@ -34,18 +38,21 @@ constexpr int UMMA_K = 16;              // K of one tcgen05.mma.kind::f16
 constexpr int EPI_THREADS = 128;        // 4 epilogue warps, one per TMEM lane quarter
 constexpr int GEMM_THREADS = 64 + EPI_THREADS;
 
-enum { EPI_STORE_BF16 = 0, EPI_ATOMIC_UPPER_F32 = 1 };
+enum { EPI_STORE_BF16 = 0, EPI_ATOMIC_UPPER_F32 = 1, EPI_STORE_BF16_T = 2, EPI_SPLIT_BF16_T = 3 };
 
 struct TcGemmArgs {
     int rows, cols;        // output extent
     int kblocks;           // 64-wide blocks along the reduction
     int tiles_n;           // column tiles (row-major tile grid when tile_list == nullptr)
     int num_tiles;         // output tiles
-    int ksplit;            // reduction splits per tile (EPI_ATOMIC_UPPER_F32 only)
+    int ksplit;            // reduction splits per tile (EPI_ATOMIC_UPPER_F32, EPI_SPLIT_BF16_T)
     int kb_per_split;
     const int2* tile_list; // (tile row, tile col) pairs, or nullptr
     void* out;
     int64_t ldo;
+    // EPI_SPLIT_BF16_T: fp32 partial of split s, row r at part[(s * rows + r) * ld_part]
+    float* part;
+    int64_t ld_part;
     int* status;
     uint64_t wait_limit_ns;
 };
@@ -266,7 +273,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                             if (col0 + i < args.cols)
                                 out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
                     }
-                } else {
+                } else if (EPI == EPI_ATOMIC_UPPER_F32) {
                     float* out_row =
                         reinterpret_cast<float*>(args.out) + static_cast<int64_t>(row) * args.ldo;
 #pragma unroll
@@ -274,6 +281,22 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                         const int col = col0 + i;
                         if (col < args.cols && col >= row) atomicAdd(out_row + col, __uint_as_float(v[i]));
                     }
+                } else if (EPI == EPI_STORE_BF16_T) {
+                    // out[col][row]: the warp's 32 lanes hold 32 consecutive rows
+                    __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(args.out) + row;
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        if (col0 + i < args.cols)
+                            o[static_cast<int64_t>(col0 + i) * args.ldo] = __float2bfloat16_rn(__uint_as_float(v[i]));
+                } else {
+                    // this split's fp32 partial (columns up to the next multiple of 32)
+                    const int split = item - (item / args.ksplit) * args.ksplit;
+                    float4* dst = reinterpret_cast<float4*>(
+                        args.part + (static_cast<int64_t>(split) * args.rows + row) * args.ld_part + col0);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
+                                             __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
                 }
             }
             tc_fence_before_sync();
@@ -880,6 +903,100 @@ cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ld
     const int grid = std::min(a.num_tiles, dev->num_sms);
     if (wide) return launch_kernel<256, 4, false, EPI_STORE_BF16>(ma, mb, a, grid, stream);
     return launch_kernel<128, 6, false, EPI_STORE_BF16>(ma, mb, a, grid, stream);
+}
+
+// Swapped product for few tokens: tiles of 128 weight rows x 128 (ntok <= 128) or 256
+// tokens. When the tiles would leave more than half of the SMs idle, the reduction splits
+// over CTAs: about one work item per SM, at least 4 k-blocks per split.
+SwapPlan gemm_swap_plan(int rows, int ntok, int kdim, int num_sms, bool allow_split)
+{
+    SwapPlan pl;
+    pl.bn = ntok <= 128 ? 128 : 256;
+    pl.tiles = ((rows + BM - 1) / BM) * ((ntok + pl.bn - 1) / pl.bn);
+    pl.kblocks = (kdim + BK - 1) / BK;
+    pl.ksplit = 1;
+    pl.kb_per_split = pl.kblocks;
+    if (allow_split && pl.tiles < num_sms / 2) {
+        const int want = std::max(1, num_sms / pl.tiles);
+        pl.kb_per_split = std::min(pl.kblocks, std::max(4, (pl.kblocks + want - 1) / want));
+        pl.ksplit = (pl.kblocks + pl.kb_per_split - 1) / pl.kb_per_split;
+    }
+    pl.ld_part = (ntok + 31) / 32 * 32;
+    pl.part_elems = pl.ksplit > 1 ? static_cast<int64_t>(pl.ksplit) * rows * pl.ld_part : 0;
+    return pl;
+}
+
+// out[n][r] = bf16(sum over s, in order, of part[(s * rows + r) * ld_part + n]). A block of
+// 32 x 32 threads takes 32 rows x 32 tokens, one output each: the partials are read along
+// tokens and the bf16 results written along rows, both coalesced, through shared memory.
+__global__ void __launch_bounds__(1024) reduce_splits_kernel(const float* __restrict__ part, int ksplit, int rows,
+                                                             int64_t ld_part, int ntok, __nv_bfloat16* __restrict__ out,
+                                                             int64_t ldo)
+{
+    __shared__ float tile[32][33];
+    const int r0 = blockIdx.x * 32, n0 = blockIdx.y * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    float acc = 0.f;
+    if (r0 + ty < rows) {
+        const float* src = part + static_cast<int64_t>(r0 + ty) * ld_part + n0 + tx;
+        const int64_t step = static_cast<int64_t>(rows) * ld_part;
+        // four partials in flight at a time, added in split order
+        int sp = 0;
+        for (; sp + 4 <= ksplit; sp += 4) {
+            const float a0 = __ldcg(src + sp * step), a1 = __ldcg(src + (sp + 1) * step);
+            const float a2 = __ldcg(src + (sp + 2) * step), a3 = __ldcg(src + (sp + 3) * step);
+            acc += a0;
+            acc += a1;
+            acc += a2;
+            acc += a3;
+        }
+        for (; sp < ksplit; ++sp) acc += __ldcg(src + sp * step);
+    }
+    tile[ty][tx] = acc;
+    __syncthreads();
+    const int n = n0 + ty, r = r0 + tx;
+    if (n < ntok && r < rows) out[static_cast<int64_t>(n) * ldo + r] = __float2bfloat16_rn(tile[tx][ty]);
+}
+
+cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t ldx, int rows, int ntok, int kdim,
+                             void* out, int64_t ldo, float* part, cudaStream_t stream)
+{
+    if (rows <= 0 || ntok <= 0) return cudaSuccess;
+    if (ntok > 256) return cudaErrorInvalidValue;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    // without a workspace the reduction is not split
+    const SwapPlan pl = gemm_swap_plan(rows, ntok, kdim, dev->num_sms, part != nullptr);
+    CUtensorMap ma, mb;
+    if (!encode_map(&ma, W, kdim, rows, ldw, BK, BM)) return cudaErrorInvalidValue;
+    if (!encode_map(&mb, X, kdim, ntok, ldx, BK, pl.bn)) return cudaErrorInvalidValue;
+    TcGemmArgs a{};
+    a.rows = rows;
+    a.cols = ntok;
+    a.kblocks = pl.kblocks;
+    a.tiles_n = (ntok + pl.bn - 1) / pl.bn;
+    a.num_tiles = pl.tiles;
+    a.ksplit = pl.ksplit;
+    a.kb_per_split = pl.kb_per_split;
+    a.tile_list = nullptr;
+    a.out = out;
+    a.ldo = ldo;
+    a.part = part;
+    a.ld_part = pl.ld_part;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    const int grid = std::min(pl.tiles * pl.ksplit, dev->num_sms);
+    if (pl.ksplit > 1) {
+        cudaError_t e = pl.bn == 128 ? launch_kernel<128, 6, false, EPI_SPLIT_BF16_T>(ma, mb, a, grid, stream)
+                                     : launch_kernel<256, 4, false, EPI_SPLIT_BF16_T>(ma, mb, a, grid, stream);
+        if (e != cudaSuccess) return e;
+        const dim3 grid_r((rows + 31) / 32, (ntok + 31) / 32);
+        reduce_splits_kernel<<<grid_r, 1024, 0, stream>>>(part, pl.ksplit, rows, pl.ld_part, ntok,
+                                                         static_cast<__nv_bfloat16*>(out), ldo);
+        return cudaGetLastError();
+    }
+    if (pl.bn == 128) return launch_kernel<128, 6, false, EPI_STORE_BF16_T>(ma, mb, a, grid, stream);
+    return launch_kernel<256, 4, false, EPI_STORE_BF16_T>(ma, mb, a, grid, stream);
 }
 
 namespace {

@@ -55,7 +55,8 @@ def make_layer(K, M, N, seed, outliers=None, sigma=0.5):
 # ------------------------------------------------------------------------------ dense (Eq. 1)
 
 @pytest.mark.parametrize("N,K,M", [(128, 512, 512), (200, 520, 264), (1, 64, 8), (300, 1024, 776),
-                                   (129, 136, 392), (9, 136, 392), (32, 520, 264), (5, 4096, 12288)])
+                                   (129, 136, 392), (9, 136, 392), (32, 520, 264), (5, 4096, 12288),
+                                   (33, 2056, 1000), (256, 1024, 776)])
 def test_dense_forward_matches_oracle(esp, N, K, M):
     _, X, W = make_layer(K, M, N, seed=100 + N)
     Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
@@ -110,6 +111,12 @@ FORWARD_CASES = [
     (600, 1024, 1000, 512, 3),     # the same on two launches
     (1000, 2048, 2312, 1000, 1),   # fused, ragged N / L / M, several row blocks
     (300, 1024, 3000, 300, 3),
+    # few tokens on tcgen05 with the weights as the 128-row operand; split reductions
+    (100, 4096, 776, 2048, 1),     # both products split (16 and 7 weight tiles)
+    (33, 1040, 3000, 600, 0),      # ragged N, K (not a multiple of 64), L and M
+    (256, 2048, 1000, 1000, 0),    # 256-token tiles
+    (129, 520, 264, 100, 1),       # 256-token tile, ragged
+    (7, 1024, 776, 448, 1),        # fewer tokens than one MMA's rows
 ]
 
 
@@ -122,7 +129,9 @@ def test_launch_counts(esp):
         assert esp.espace_linear_forward_launches(p, 1) == 1          # decode kernel
         assert esp.espace_linear_forward_launches(p, 600) == 1        # fused
         assert esp.espace_linear_forward_launches(p, 600, esp.PATH_TENSOR_SPLIT) == 2
-        assert esp.espace_linear_forward_launches(p, 100, esp.PATH_TENSOR) == 2
+        # few tokens: both products split their reduction here (4 and 8 weight tiles), each
+        # followed by the launch that adds the partials
+        assert esp.espace_linear_forward_launches(p, 100, esp.PATH_TENSOR) == 4
         assert esp.espace_linear_forward_launches(p, 64, esp.PATH_SMALL_N) == -1
     finally:
         esp.espace_proj_destroy(p)
@@ -141,6 +150,28 @@ def test_linear_forward_matches_oracle(esp, N, K, M, L, path):
         esp.espace_check()
         Y_o, _, _ = oracle.forward(f64(X), oracle.bf16_round(P), f64(W))
         assert_y_close(Y, Y_o)
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+def test_few_token_forward_is_reproducible(esp):
+    """The split reductions add their fp32 partials in a fixed order: two calls give the
+    same bits."""
+    N, K, M, L = 96, 4096, 1000, 2048
+    _, X, W = make_layer(K, M, N, seed=31)
+    P = synth.random_projection(K, L, seed=31)
+    p = esp.espace_proj_from_host(P, dev(W))
+    try:
+        Xd = dev(X)
+        Y1 = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        Y2 = torch.empty_like(Y1)
+        esp.espace_linear_forward(p, Xd, Y1)
+        esp.espace_linear_forward(p, Xd, Y2)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        assert torch.equal(Y1.view(torch.int16), Y2.view(torch.int16))
+        Y_o, _, _ = oracle.forward(f64(X), oracle.bf16_round(P), f64(W))
+        assert_y_close(Y1, Y_o)
     finally:
         esp.espace_proj_destroy(p)
 
