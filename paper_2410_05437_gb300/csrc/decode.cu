@@ -12,10 +12,14 @@
 // consumed, phase 1 then phase 2, and copies each row piece into a ring of shared-memory
 // stages with 1-D bulk copies (cp.async.bulk) completing on the stage's mbarrier. The
 // producer does not wait for the grid barrier: while the consumers wait for Z, it keeps
-// filling the ring with W'^T rows, so HBM stays busy across the barrier.
+// filling the ring with W'^T rows, so HBM stays busy across the barrier. (Holding the W'^T
+// copies back until phase 1 has landed was measured slower: they then arrive as one burst
+// just when the barrier's few L2 round trips are on the critical path.)
 //
 // Compute. The 16 consumer warps form groups of WPS warps (8 for N <= 8, 16 above); group q
-// takes stages q, q + 16/WPS, ..., and its warps split the stage's k-block
+// takes stages q, q + 16/WPS, .... For the dense product of one token, warp u of a group
+// owns row u of each stage and runs fp32 FMA against the token, copied once to shared
+// memory; otherwise the group's warps split the stage's k-block
 // into 32-wide chunks. Each warp runs mma.sync.m16n8k16 (bf16 in, fp32 accumulate) with the
 // tokens as the A operand (16 rows, rows >= N zero) and the 8 streamed rows as the B
 // operand, one accumulator per chunk so consecutive MMAs do not wait on each other. The
@@ -66,6 +70,7 @@ struct DecodeArgs {
     int nt;
     int stages;                  // ring depth
     int acc_rows;                // rows of the shared accumulator
+    int tok_elems;               // one token (N = 1): bf16 values of its shared-memory copy
     unsigned int* bar;           // grid barrier counter
     int* status;
     uint64_t wait_limit_ns;
@@ -154,7 +159,7 @@ struct DecodeCfg {
     static constexpr int SK = 2048;                           // k-block of one stage
     // consumer warps per stage: each group of WPS warps takes every NG-th stage and splits its
     // k-block; wider token tiles use larger groups so the fragments fit the register budget
-    static constexpr int WPS = HI ? 16 : 8;
+    static constexpr int WPS = (HI && MT > 0) ? 16 : 8;
     static constexpr int NG = DEC_CWARPS / WPS;
     static constexpr int CPW = SK / 32 / WPS;                 // 32-wide chunks per warp and stage
     static constexpr int NACC = MT == 2 ? 1 : CPW < 4 ? CPW : 4;   // independent MMA accumulators
@@ -162,13 +167,19 @@ struct DecodeCfg {
     static constexpr int STAGE_BYTES = DEC_ROWS * PITCH;
     // accumulator row pitch (floats): 16 tokens per m16 tile plus 4, so the lanes of one
     // flush (rows 2t, 2t+1; tokens g) hit 32 different banks
-    static constexpr int NTP = 16 * MT + 4;
+    static constexpr int NTP = MT == 0 ? 1 : 16 * MT + 4;
 };
 
 // A warp's token fragments for one k-block: v[chunk][m16 tile][row g / row g + 8].
 template <int MT, bool HI>
 struct TokFrag {
     uint4 v[DecodeCfg<MT, HI>::CPW][MT][HI ? 2 : 1];
+};
+// One token (MT = 0): lane l holds the token's fp32 values at k = 256 c + 8 l + e of the
+// k-block, x[8 c + e].
+template <>
+struct TokFrag<0, false> {
+    float x[64];
 };
 
 // Stage layout. When one k-block covers whole rows (kdim <= SK), a stage's rows are
@@ -186,6 +197,23 @@ __device__ __forceinline__ void load_tokens(TokFrag<MT, HI>& T, const __nv_bfloa
                                             int nt, int kb, int u, int g, int t)
 {
     using C = DecodeCfg<MT, HI>;
+    if constexpr (MT == 0) {
+        // B is the CTA's shared-memory copy of the token here
+        const int lane = g * 4 + t;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            const int k = kb * C::SK + 256 * c + 8 * lane;
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (k < kdim) v = *reinterpret_cast<const uint4*>(B + k);
+            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                T.x[8 * c + 2 * e] = __uint_as_float(w[e] << 16);
+                T.x[8 * c + 2 * e + 1] = __uint_as_float(w[e] & 0xffff0000u);
+            }
+        }
+        return;
+    } else {
 #pragma unroll
     for (int c = 0; c < C::CPW; ++c) {
         const int k = kb * C::SK + 32 * (u * C::CPW + c) + 8 * t;
@@ -203,6 +231,7 @@ __device__ __forceinline__ void load_tokens(TokFrag<MT, HI>& T, const __nv_bfloa
             }
         }
     }
+    }
 }
 
 // One stage for the warp with k-part u: the MMAs over its chunks, release of the stage, and
@@ -213,6 +242,36 @@ __device__ __forceinline__ void consume_stage(const unsigned char* st, uint64_t*
                                               int lane)
 {
     using C = DecodeCfg<MT, HI>;
+    if constexpr (MT == 0) {
+        // one token: warp u owns row u of the stage and reads it 512 contiguous bytes at a
+        // time; fp32 FMA into four accumulators, then one warp reduction per row
+        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+        if (u < rows) {
+            const unsigned char* rp = st + stage_row_offset<C::PITCH>(u, ksz, whole);
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const int kl = 256 * c + 8 * lane;
+                if (kl < ksz) {
+                    const uint4 w = *reinterpret_cast<const uint4*>(rp + kl * 2);
+                    s0 = fmaf(__uint_as_float(w.x << 16), T.x[8 * c + 0], s0);
+                    s1 = fmaf(__uint_as_float(w.x & 0xffff0000u), T.x[8 * c + 1], s1);
+                    s2 = fmaf(__uint_as_float(w.y << 16), T.x[8 * c + 2], s2);
+                    s3 = fmaf(__uint_as_float(w.y & 0xffff0000u), T.x[8 * c + 3], s3);
+                    s0 = fmaf(__uint_as_float(w.z << 16), T.x[8 * c + 4], s0);
+                    s1 = fmaf(__uint_as_float(w.z & 0xffff0000u), T.x[8 * c + 5], s1);
+                    s2 = fmaf(__uint_as_float(w.w << 16), T.x[8 * c + 6], s2);
+                    s3 = fmaf(__uint_as_float(w.w & 0xffff0000u), T.x[8 * c + 7], s3);
+                }
+            }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty_bar);
+        float sum = (s0 + s1) + (s2 + s3);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        if (lane == 0 && u < rows) atomicAdd(acc + (r0l + u) * C::NTP, sum);
+        return;
+    } else {
     const int g = lane >> 2, t = lane & 3;
     st += stage_row_offset<C::PITCH>(g, ksz, whole);
     float d[C::NACC][MT][4];
@@ -257,6 +316,7 @@ __device__ __forceinline__ void consume_stage(const unsigned char* st, uint64_t*
             if (r_hi) atomicAdd(a + C::NTP + n + 8, d[0][mt][3]);
         }
     }
+    }
 }
 
 template <int MT, bool HI>
@@ -274,7 +334,9 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
 
 
     float* acc = reinterpret_cast<float*>(smem);
-    unsigned char* ring = smem + ((static_cast<size_t>(a.acc_rows) * C::NTP * 4 + 127) & ~static_cast<size_t>(127));
+    const size_t acc_bytes = (static_cast<size_t>(a.acc_rows) * C::NTP * 4 + 127) & ~static_cast<size_t>(127);
+    __nv_bfloat16* tok_s = reinterpret_cast<__nv_bfloat16*>(smem + acc_bytes);
+    unsigned char* ring = smem + acc_bytes + ((static_cast<size_t>(a.tok_elems) * 2 + 127) & ~static_cast<size_t>(127));
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < a.stages; ++s) {
@@ -349,6 +411,16 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
         const int nkb = (kdim + C::SK - 1) / C::SK;
         const int nrs = (rb1[p] - rb0[p] + DEC_ROWS - 1) / DEC_ROWS;   // row stages per k-block
         // stages run k-block-major; this group takes stages group, group + NG, ...
+        if constexpr (MT == 0) {
+            // one token: copy it to shared memory once (one 16-byte load per thread and
+            // round), so that each warp reads it from there rather than from L2
+            for (int k = 8 * threadIdx.x; k < kdim; k += 8 * DEC_CWARPS * 32) {
+                const uint4* src = reinterpret_cast<const uint4*>(B + k);
+                *reinterpret_cast<uint4*>(tok_s + k) = coherent ? __ldcg(src) : __ldg(src);
+            }
+            consumer_sync();
+            B = tok_s;
+        }
         TokFrag<MT, HI> T;
         int cur_kb = -1;
         for (int i = group; i < nkb * nrs; i += C::NG) {
@@ -400,11 +472,12 @@ struct DecodePlan {
     bool hi = false;
     int stages = 0;
     int acc_rows = 0;
+    int tok_elems = 0;
     int smem = 0;
     int cut[2][DEC_MAX_GRID + 1] = {};
 };
 
-int ntp_of(int mt) { return 16 * mt + 4; }
+int ntp_of(int mt) { return mt == 0 ? 1 : 16 * mt + 4; }
 int stage_bytes_of(int) { return DecodeCfg<1, false>::STAGE_BYTES; }
 
 bool compute_plan(int mt, int phases, int R0, int k0, int R1, int k1, int G, DecodePlan* pl)
@@ -418,10 +491,13 @@ bool compute_plan(int mt, int phases, int R0, int k0, int R1, int k1, int G, Dec
     if (static_cast<int64_t>(max_rows) * ntp_of(mt) * 4 > DEC_SMEM_LIMIT) return false;
     pl->acc_rows = max_rows;
     const int acc_bytes = (pl->acc_rows * ntp_of(mt) * 4 + 127) & ~127;
+    // one token: its shared-memory copy, for the longer of the two reductions
+    pl->tok_elems = mt == 0 ? std::max(k0, phases > 1 ? k1 : 0) : 0;
+    const int tok_bytes = (pl->tok_elems * 2 + 127) & ~127;
     const int sb = stage_bytes_of(mt);
-    pl->stages = std::min(DEC_MAX_STAGES, (DEC_SMEM_LIMIT - 1024 - acc_bytes) / sb);
+    pl->stages = std::min(DEC_MAX_STAGES, (DEC_SMEM_LIMIT - 1024 - acc_bytes - tok_bytes) / sb);
     if (pl->stages < DEC_MIN_STAGES) return false;
-    pl->smem = acc_bytes + pl->stages * sb;
+    pl->smem = acc_bytes + tok_bytes + pl->stages * sb;
     return true;
 }
 
@@ -432,7 +508,9 @@ bool make_plan(int nt, int phases, int R0, int k0, int R1, int k1, int G, Decode
     if (k0 < 8 || k0 % 8 != 0 || R0 < 1) return false;
     if (phases > 1 && (k1 < 8 || k1 % 8 != 0 || R1 < 1)) return false;
     if (phases < 2) R1 = k1 = 0;
-    const int mt = nt <= 16 ? 1 : 2;
+    // one token, one phase (the dense product): fp32 FMA with the token in shared memory; the
+    // projected layer's two phases measured faster on the MMA path for one token too
+    const int mt = (nt == 1 && phases == 1 && k0 <= 16384) ? 0 : nt <= 16 ? 1 : 2;
     struct Entry {
         bool valid = false, ok = false;
         int key[7] = {};
@@ -479,6 +557,7 @@ cudaError_t launch_t(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev,
     }
     a.stages = pl.stages;
     a.acc_rows = pl.acc_rows;
+    a.tok_elems = pl.tok_elems;
     std::copy(&pl.cut[0][0], &pl.cut[0][0] + 2 * (DEC_MAX_GRID + 1), &a.cut[0][0]);
     if (a.phases == 1) {
         // no grid barrier: an ordinary launch
@@ -492,6 +571,7 @@ cudaError_t launch_t(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev,
 
 cudaError_t launch_any(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev, cudaStream_t stream)
 {
+    if (pl.mt == 0) return launch_t<0, false>(a, pl, dev, stream);
     if (pl.mt == 2) return launch_t<2, true>(a, pl, dev, stream);
     if (pl.hi) return launch_t<1, true>(a, pl, dev, stream);
     return launch_t<1, false>(a, pl, dev, stream);
