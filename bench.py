@@ -417,7 +417,8 @@ def side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, espa
             "espace_gbs": ebytes / e_us / 1e3, "espace_frac_hbm": ebytes / e_us / 1e3 / peak_hbm,
             "espace_tflops": 2.0 * n_tok * (K * L + L * M) / e_us / 1e6,
             "dense_gbs": dbytes / d_us / 1e3,
-            "path": "decode kernel" if esp.espace_linear_forward_launches(sets[0]["p"], n_tok) == 1 and n_tok <= 32 else "tcgen05"}
+            "path": ("decode kernel" if esp.espace_linear_forward_launches(sets[0]["p"], n_tok) == 1 and n_tok <= 32
+                     else "tcgen05")}
     rows["decode_sweep_llama2_qkv"] = sweep
     return rows
 

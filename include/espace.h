@@ -146,7 +146,7 @@ void espace_proj_destroy(espace_proj_t p);
 
 /* Async. Y = (P^T W)^T (P^T X) for the N tokens of X_dev ([N][K] bf16) into Y_dev
  * ([N][M] bf16): Z = X P is accumulated in fp32 and rounded to bf16 (the paper computes in
- * BF16, Sec. A.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 32 runs
+ * BF16, Sec. A.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 16 runs
  * a bandwidth-bound kernel that streams P and W' once; N <= 256 runs two tcgen05 launches
  * with the weights as the 128-row operand (phase 1 splits its reduction over the SMs and
  * adds the fp32 partials in a fixed order, so results are reproducible bit for bit);
@@ -199,7 +199,7 @@ int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev, int64_t N,
 
 /* Async. The uncompressed layer of Eq. 1, Y = W^T X, as Y_dev[N][M] = X_dev[N][K] W_dev^T
  * with W_dev in [M][K] layout, with fp32 accumulation and bf16 output on the same kernel
- * families as the projected layer (N <= 32: the streaming kernel; N <= 256: tcgen05 with
+ * families as the projected layer (N <= 8: the streaming kernel; N <= 256: tcgen05 with
  * the weights as the 128-row operand, no split; above: tcgen05): the baseline the
  * projected layer is measured against. */
 int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev,

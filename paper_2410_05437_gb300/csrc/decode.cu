@@ -71,6 +71,7 @@ struct DecodeArgs {
     int stages;                  // ring depth
     int acc_rows;                // rows of the shared accumulator
     int tok_elems;               // one token (N = 1): bf16 values of its shared-memory copy
+    int slot_floats;             // 16-warp groups: floats of the partial-sum slots
     unsigned int* bar;           // grid barrier counter
     int* status;
     uint64_t wait_limit_ns;
@@ -168,6 +169,11 @@ struct DecodeCfg {
     // accumulator row pitch (floats): 16 tokens per m16 tile plus 4, so the lanes of one
     // flush (rows 2t, 2t+1; tokens g) hit 32 different banks
     static constexpr int NTP = MT == 0 ? 1 : 16 * MT + 4;
+    // two token tiles (N > 16): a stage's partial sums meet through per-warp slots in shared
+    // memory (double-buffered, [warp][8 rows][NTP]) instead of contended atomics (measured
+    // faster there, slower for one tile)
+    static constexpr bool SLOTS = MT == 2;
+    static constexpr int SLOT_FLOATS = SLOTS ? 2 * 16 * DEC_ROWS * NTP : 0;
 };
 
 // A warp's token fragments for one k-block: v[chunk][m16 tile][row g / row g + 8].
@@ -239,7 +245,7 @@ __device__ __forceinline__ void load_tokens(TokFrag<MT, HI>& T, const __nv_bfloa
 template <int MT, bool HI>
 __device__ __forceinline__ void consume_stage(const unsigned char* st, uint64_t* empty_bar, const TokFrag<MT, HI>& T,
                                               int ksz, bool whole, int rows, int r0l, int nt, float* acc, int u,
-                                              int lane)
+                                              int lane, float* slot)
 {
     using C = DecodeCfg<MT, HI>;
     if constexpr (MT == 0) {
@@ -300,8 +306,21 @@ __device__ __forceinline__ void consume_stage(const unsigned char* st, uint64_t*
         for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
             for (int e = 0; e < 4; ++e) d[0][mt][e] += d[q][mt][e];
-    // d[0][mt]: {token g, rows 2t, 2t+1}, {token g+8, rows 2t, 2t+1}; rows past the CTA's range
-    // were not copied and are not flushed
+    // d[0][mt]: {token g, rows 2t, 2t+1}, {token g+8, rows 2t, 2t+1}
+    if constexpr (C::SLOTS) {
+        // this warp's slot; the rows and tokens that count are picked when the slots are summed
+        float* sl = slot + (u * DEC_ROWS + 2 * t) * C::NTP;
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+            const int n = mt * 16 + g;
+            sl[n] = d[0][mt][0];
+            sl[C::NTP + n] = d[0][mt][1];
+            sl[n + 8] = d[0][mt][2];
+            sl[C::NTP + n + 8] = d[0][mt][3];
+        }
+        return;
+    }
+    // rows past the CTA's range were not copied and are not flushed
     const bool r_lo = 2 * t < rows, r_hi = 2 * t + 1 < rows;
     float* a = acc + (r0l + 2 * t) * C::NTP;
 #pragma unroll
@@ -336,7 +355,10 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
     float* acc = reinterpret_cast<float*>(smem);
     const size_t acc_bytes = (static_cast<size_t>(a.acc_rows) * C::NTP * 4 + 127) & ~static_cast<size_t>(127);
     __nv_bfloat16* tok_s = reinterpret_cast<__nv_bfloat16*>(smem + acc_bytes);
-    unsigned char* ring = smem + acc_bytes + ((static_cast<size_t>(a.tok_elems) * 2 + 127) & ~static_cast<size_t>(127));
+    const size_t tok_bytes = (static_cast<size_t>(a.tok_elems) * 2 + 127) & ~static_cast<size_t>(127);
+    float* slots = reinterpret_cast<float*>(smem + acc_bytes + tok_bytes);
+    unsigned char* ring = smem + acc_bytes + tok_bytes +
+                          ((static_cast<size_t>(a.slot_floats) * 4 + 127) & ~static_cast<size_t>(127));
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < a.stages; ++s) {
@@ -431,14 +453,31 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
             }
             const int j = j0 + i;
             const int slot = j % a.stages;
-            if (*abort) continue;
-            if (!mbar_wait(&full[slot], static_cast<uint32_t>(j / a.stages) & 1u, abort, a.status, a.wait_limit_ns,
-                           ESPACE_ERR_TIMEOUT))
-                continue;
             const int r0l = rs * DEC_ROWS;
-            consume_stage<MT, HI>(ring + static_cast<size_t>(slot) * C::STAGE_BYTES, &empty[slot], T,
-                                  min(C::SK, kdim - kb * C::SK), kdim <= C::SK, min(DEC_ROWS, rb1[p] - rb0[p] - r0l),
-                                  r0l, a.nt, acc, u, lane);
+            const int srows = min(DEC_ROWS, rb1[p] - rb0[p] - r0l);
+            float* slot_buf = slots + (i & 1) * (C::SLOT_FLOATS / 2);
+            const bool ok = !*abort && mbar_wait(&full[slot], static_cast<uint32_t>(j / a.stages) & 1u, abort,
+                                                 a.status, a.wait_limit_ns, ESPACE_ERR_TIMEOUT);
+            if (ok)
+                consume_stage<MT, HI>(ring + static_cast<size_t>(slot) * C::STAGE_BYTES, &empty[slot], T,
+                                      min(C::SK, kdim - kb * C::SK), kdim <= C::SK, srows, r0l, a.nt, acc, u, lane,
+                                      slot_buf);
+            if constexpr (C::SLOTS) {
+                // every consumer warp takes every stage (one group): one barrier per stage,
+                // reached by all of them whatever happened above; then one thread per
+                // (row, token) adds the 16 warps' slots in warp order (the double buffer lets
+                // the next stage's slots be written before everyone has read these)
+                consumer_sync();
+                if (!*abort) {
+                    const int e = threadIdx.x, r = e / C::NTP, n = e - r * C::NTP;
+                    if (e < DEC_ROWS * C::NTP && r < srows && n < a.nt) {
+                        float sum = 0.f;
+#pragma unroll
+                        for (int w = 0; w < DEC_CWARPS; ++w) sum += slot_buf[(w * DEC_ROWS + r) * C::NTP + n];
+                        acc[(r0l + r) * C::NTP + n] += sum;
+                    }
+                }
+            }
         }
         j0 += nkb * nrs;
         consumer_sync();
@@ -473,6 +512,7 @@ struct DecodePlan {
     int stages = 0;
     int acc_rows = 0;
     int tok_elems = 0;
+    int slot_floats = 0;
     int smem = 0;
     int cut[2][DEC_MAX_GRID + 1] = {};
 };
@@ -480,9 +520,10 @@ struct DecodePlan {
 int ntp_of(int mt) { return mt == 0 ? 1 : 16 * mt + 4; }
 int stage_bytes_of(int) { return DecodeCfg<1, false>::STAGE_BYTES; }
 
-bool compute_plan(int mt, int phases, int R0, int k0, int R1, int k1, int G, DecodePlan* pl)
+bool compute_plan(int mt, bool hi, int phases, int R0, int k0, int R1, int k1, int G, DecodePlan* pl)
 {
     pl->mt = mt;
+    pl->hi = hi;
     decode_cuts(G, phases, R0, k0, phases > 1 ? R1 : 0, phases > 1 ? k1 : 1, pl->cut[0], pl->cut[1]);
     int max_rows = 1;
     for (int b = 0; b < G; ++b)
@@ -494,10 +535,12 @@ bool compute_plan(int mt, int phases, int R0, int k0, int R1, int k1, int G, Dec
     // one token: its shared-memory copy, for the longer of the two reductions
     pl->tok_elems = mt == 0 ? std::max(k0, phases > 1 ? k1 : 0) : 0;
     const int tok_bytes = (pl->tok_elems * 2 + 127) & ~127;
+    pl->slot_floats = mt == 2 ? 2 * 16 * DEC_ROWS * ntp_of(mt) : 0;
+    const int slot_bytes = (pl->slot_floats * 4 + 127) & ~127;
     const int sb = stage_bytes_of(mt);
-    pl->stages = std::min(DEC_MAX_STAGES, (DEC_SMEM_LIMIT - 1024 - acc_bytes - tok_bytes) / sb);
+    pl->stages = std::min(DEC_MAX_STAGES, (DEC_SMEM_LIMIT - 1024 - acc_bytes - tok_bytes - slot_bytes) / sb);
     if (pl->stages < DEC_MIN_STAGES) return false;
-    pl->smem = acc_bytes + tok_bytes + pl->stages * sb;
+    pl->smem = acc_bytes + tok_bytes + slot_bytes + pl->stages * sb;
     return true;
 }
 
@@ -511,31 +554,30 @@ bool make_plan(int nt, int phases, int R0, int k0, int R1, int k1, int G, Decode
     // one token, one phase (the dense product): fp32 FMA with the token in shared memory; the
     // projected layer's two phases measured faster on the MMA path for one token too
     const int mt = (nt == 1 && phases == 1 && k0 <= 16384) ? 0 : nt <= 16 ? 1 : 2;
+    const bool hi = mt > 0 && nt > 8;
     struct Entry {
         bool valid = false, ok = false;
-        int key[7] = {};
+        int key[8] = {};
         DecodePlan plan;
     };
     static Entry cache[16];
     static int next = 0;
     static std::mutex mu;
-    const int key[7] = {mt, phases, R0, k0, R1, k1, G};
+    const int key[8] = {mt, hi ? 1 : 0, phases, R0, k0, R1, k1, G};
     std::lock_guard<std::mutex> lock(mu);
     for (Entry& e : cache)
-        if (e.valid && std::equal(key, key + 7, e.key)) {
+        if (e.valid && std::equal(key, key + 8, e.key)) {
             if (!e.ok) return false;
             *plan = e.plan;
-            plan->hi = nt > 8;
             return true;
         }
     Entry& e = cache[next];
     next = (next + 1) % 16;
     e.valid = true;
-    std::copy(key, key + 7, e.key);
-    e.ok = compute_plan(mt, phases, R0, k0, R1, k1, G, &e.plan);
+    std::copy(key, key + 8, e.key);
+    e.ok = compute_plan(mt, hi, phases, R0, k0, R1, k1, G, &e.plan);
     if (!e.ok) return false;
     *plan = e.plan;
-    plan->hi = nt > 8;
     return true;
 }
 
@@ -558,6 +600,7 @@ cudaError_t launch_t(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev,
     a.stages = pl.stages;
     a.acc_rows = pl.acc_rows;
     a.tok_elems = pl.tok_elems;
+    a.slot_floats = pl.slot_floats;
     std::copy(&pl.cut[0][0], &pl.cut[0][0] + 2 * (DEC_MAX_GRID + 1), &a.cut[0][0]);
     if (a.phases == 1) {
         // no grid barrier: an ordinary launch

@@ -628,7 +628,7 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
     const bool small_ok = N <= DECODE_MAX_TOKENS && decode_supported(n, K, Lp, M, dev->num_sms);
     if (path == ESPACE_PATH_SMALL_N && !small_ok)
         return fail(ESPACE_ERR_SHAPE, "espace_linear_forward: N=%lld (K=%d, Lp=%d) beyond the small-N kernels", (long long)N, K, Lp);
-    const bool small = path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok);
+    const bool small = path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok && N <= DECODE_AUTO_TOKENS);
     DeviceGuard g(p->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int rc = ensure_z(p, N, st);
@@ -673,7 +673,8 @@ int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path)
     const int n = static_cast<int>(N), K = static_cast<int>(p->K), M = static_cast<int>(p->M),
               Lp = static_cast<int>(p->Lp);
     const bool small_ok = N <= DECODE_MAX_TOKENS && decode_supported(n, K, Lp, M, dev->num_sms);
-    if (path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok)) return small_ok ? 1 : -1;
+    if (path == ESPACE_PATH_SMALL_N || (path == ESPACE_PATH_AUTO && small_ok && N <= DECODE_AUTO_TOKENS))
+        return small_ok ? 1 : -1;
     if (swap_forward_applies(n, path)) {
         // one launch per product, plus one per split reduction
         const int a = gemm_swap_plan(Lp, n, K, dev->num_sms, true).ksplit > 1 ? 2 : 1;
@@ -703,7 +704,8 @@ int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_
     int rc = device_info(&dev);
     if (rc != ESPACE_OK) return rc;
     // few tokens: stream W once through the decode kernel; otherwise the tcgen05 GEMM
-    if (N <= DECODE_MAX_TOKENS && decode_dense_supported(static_cast<int>(N), static_cast<int>(K), static_cast<int>(M), dev->num_sms)) {
+    if (N <= DECODE_DENSE_AUTO_TOKENS &&
+        decode_dense_supported(static_cast<int>(N), static_cast<int>(K), static_cast<int>(M), dev->num_sms)) {
         CUDA_TRY(launch_decode_dense(W_dev, X_dev, Y_dev, static_cast<int>(K), static_cast<int>(M), static_cast<int>(N),
                                      static_cast<cudaStream_t>(stream)),
                  "espace_dense_forward: decode launch");

@@ -51,8 +51,11 @@ bool pair_kernel_enabled();
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
 
-// Token counts served by the decode kernels.
+// Token counts served by the decode kernels (when asked for), and chosen for them by the
+// automatic paths: above these, the swapped tcgen05 products measured faster.
 constexpr int DECODE_MAX_TOKENS = 32;
+constexpr int DECODE_AUTO_TOKENS = 16;
+constexpr int DECODE_DENSE_AUTO_TOKENS = 8;
 
 // Decode-shaped forward (nt <= DECODE_MAX_TOKENS) in one cooperative launch: Z[nt][Lp] = X P
 // from P^T [Lp][K], a grid barrier, then Y[nt][M] = Z W' from W'^T [M][Lp]; each matrix

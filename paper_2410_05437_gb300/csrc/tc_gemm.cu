@@ -53,6 +53,10 @@ struct TcGemmArgs {
     // EPI_SPLIT_BF16_T: fp32 partial of split s, row r at part[(s * rows + r) * ld_part]
     float* part;
     int64_t ld_part;
+    // K-major only: rows of each B tile load (0: BN). Fewer than BN when B has fewer rows:
+    // the tile's other rows keep stale shared memory, which reaches only output columns past
+    // `cols` (never stored) -- cheaper than the copy engine's zero fill of absent rows
+    int b_rows;
     int* status;
     uint64_t wait_limit_ns;
 };
@@ -156,7 +160,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                     }
                     uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
                     uint8_t* sb = sa + Cfg::A_BYTES;
-                    mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
+                    mbar_arrive_expect_tx(&full[stage], (!MN_MAJOR && args.b_rows > 0)
+                                                            ? static_cast<uint32_t>(Cfg::A_BYTES + args.b_rows * BK * 2)
+                                                            : static_cast<uint32_t>(Cfg::STAGE_BYTES));
                     if (MN_MAJOR) {
                         // 64 features x 64 tokens per box; box h of a tile at +h*8 KB
                         tma_load_2d(sa, &map_a, &full[stage], tm * BM, kb * BK);
@@ -967,9 +973,11 @@ cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t 
     if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
     // without a workspace the reduction is not split
     const SwapPlan pl = gemm_swap_plan(rows, ntok, kdim, dev->num_sms, part != nullptr);
+    // token tiles load only the rows that exist (rounded up to 8)
+    const int b_rows = std::min(pl.bn, (ntok + 7) / 8 * 8);
     CUtensorMap ma, mb;
     if (!encode_map(&ma, W, kdim, rows, ldw, BK, BM)) return cudaErrorInvalidValue;
-    if (!encode_map(&mb, X, kdim, ntok, ldx, BK, pl.bn)) return cudaErrorInvalidValue;
+    if (!encode_map(&mb, X, kdim, ntok, ldx, BK, b_rows)) return cudaErrorInvalidValue;
     TcGemmArgs a{};
     a.rows = rows;
     a.cols = ntok;
@@ -983,6 +991,7 @@ cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t 
     a.ldo = ldo;
     a.part = part;
     a.ld_part = pl.ld_part;
+    a.b_rows = b_rows;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
     const int grid = std::min(pl.tiles * pl.ksplit, dev->num_sms);
