@@ -294,6 +294,9 @@ def run_ours(args, world, rank, local):
     if not args.no_rows:
         rows = side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, ms_per_step)
     clocks = sampler.stop()
+    if not args.no_rows and rank == 0:
+        # the other workloads (after the clock sampler: they are not part of the timed step)
+        rows.update(config_rows(esp, peak_tc, peak_hbm))
 
     fused = esp.espace_linear_forward_launches(sets[0]["p"], N) == 1
     if fused:
@@ -394,32 +397,143 @@ def side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, espa
                                 "frac_tensor_peak": cflops / cal_ms / 1e9 / peak_tc}
     esp.espace_calib_destroy(h)
     del Xc
-    # decode-shaped forward, N = 1 .. 512 tokens: ESPACE and dense, each replayed from a
-    # CUDA graph of 20 calls so that host launch overhead is not in the GPU time
+    # decode-shaped forward, N = 1 .. 512 tokens, on the main workload's rotating sets
+    rows["decode_sweep_llama2_qkv"] = decode_sweep(esp, K, M, L, 0, peak_hbm, sets=sets)
+    return rows
+
+
+def events_ms(call, reps=10, warm=3):
+    """Mean GPU time of one call, from CUDA events around `reps` calls after `warm` calls."""
+    for i in range(warm):
+        call(i)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for i in range(reps):
+        call(i)
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def device_projection(esp, K, L, W, seed):
+    """A projection handle for timing only: a seeded random bf16 P^T on the device, folded
+    with W on the device (the kernels' time depends on the shapes, not the values)."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(int(seed) % (1 << 63))
+    PT = (torch.randn((L, K), generator=gen, device="cuda") * K ** -0.5).to(torch.bfloat16)
+    p = esp.espace_proj_from_device(PT, W)
+    del PT
+    return p
+
+
+def layer_row(esp, K, M, L, N, seed, peak_tc):
+    """One layer at N tokens: the projected forward and the dense one (inputs larger than L2
+    are read by every call, so no rotation is needed)."""
+    W = synth.weights_device(M, K, seed=seed)
+    X = synth.ActivationModel(K, seed=seed).sample_device(N)
+    Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+    p = device_projection(esp, K, L, W, seed)
+    try:
+        e_ms = events_ms(lambda i: esp.espace_linear_forward(p, X, Y))
+        d_ms = events_ms(lambda i: esp.espace_dense_forward(X, W, Y))
+        esp.espace_check()
+    finally:
+        esp.espace_proj_destroy(p)
+    flops, dflops = 2.0 * N * (K * L + L * M), 2.0 * N * K * M
+    return {"K": K, "M": M, "L": L, "N": N, "espace_ms": e_ms, "dense_ms": d_ms, "speedup": d_ms / e_ms,
+            "espace_tflops": flops / e_ms / 1e9, "espace_frac_tensor_peak": flops / e_ms / 1e9 / peak_tc,
+            "dense_tflops": dflops / d_ms / 1e9}
+
+
+def decode_sweep(esp, K, M, L, seed, peak_hbm, sets=None):
+    """N = 1 .. 512 tokens, projected and dense, each replayed from a CUDA graph of 20 calls
+    rotating over four weight sets (so that no call finds its weights in L2)."""
+    own = sets is None
+    if own:
+        sets = []
+        for c in range(SETS):
+            W = synth.weights_device(M, K, seed=seed, chunk=c)
+            sets.append({"W": W, "p": device_projection(esp, K, L, W, seed + c),
+                         "X": synth.ActivationModel(K, seed=seed).sample_device(max(synth.DECODE_TOKENS), chunk=c)})
     Lp = (L + 63) // 64 * 64
     sweep = {}
-    for n_tok in synth.DECODE_TOKENS:
-        xs = [s["X"][:n_tok].contiguous() for s in sets]
-        ys = [torch.empty((n_tok, M), dtype=torch.bfloat16, device="cuda") for _ in sets]
+    try:
+        for n_tok in synth.DECODE_TOKENS:
+            xs = [s["X"][:n_tok].contiguous() for s in sets]
+            ys = [torch.empty((n_tok, M), dtype=torch.bfloat16, device="cuda") for _ in sets]
 
-        def espace_call(i, xs=xs, ys=ys):
-            esp.espace_linear_forward(sets[i % SETS]["p"], xs[i % SETS], ys[i % SETS])
+            def espace_call(i, xs=xs, ys=ys):
+                esp.espace_linear_forward(sets[i % SETS]["p"], xs[i % SETS], ys[i % SETS])
 
-        def dense_call(i, xs=xs, ys=ys):
-            esp.espace_dense_forward(xs[i % SETS], sets[i % SETS]["W"], ys[i % SETS])
+            def dense_call(i, xs=xs, ys=ys):
+                esp.espace_dense_forward(xs[i % SETS], sets[i % SETS]["W"], ys[i % SETS])
 
-        e_us = graph_time_us(espace_call)
-        d_us = graph_time_us(dense_call)
-        ebytes = 2.0 * (K * Lp + Lp * M + n_tok * (K + M))
-        dbytes = 2.0 * (K * M + n_tok * (K + M))
-        sweep[str(n_tok)] = {
-            "espace_us": e_us, "dense_us": d_us, "speedup": d_us / e_us,
-            "espace_gbs": ebytes / e_us / 1e3, "espace_frac_hbm": ebytes / e_us / 1e3 / peak_hbm,
-            "espace_tflops": 2.0 * n_tok * (K * L + L * M) / e_us / 1e6,
-            "dense_gbs": dbytes / d_us / 1e3,
-            "path": ("decode kernel" if esp.espace_linear_forward_launches(sets[0]["p"], n_tok) == 1 and n_tok <= 32
-                     else "tcgen05")}
-    rows["decode_sweep_llama2_qkv"] = sweep
+            e_us = graph_time_us(espace_call)
+            d_us = graph_time_us(dense_call)
+            ebytes = 2.0 * (K * Lp + Lp * M + n_tok * (K + M))
+            dbytes = 2.0 * (K * M + n_tok * (K + M))
+            sweep[str(n_tok)] = {
+                "espace_us": e_us, "dense_us": d_us, "speedup": d_us / e_us,
+                "espace_gbs": ebytes / e_us / 1e3, "espace_frac_hbm": ebytes / e_us / 1e3 / peak_hbm,
+                "espace_tflops": 2.0 * n_tok * (K * L + L * M) / e_us / 1e6,
+                "dense_gbs": dbytes / d_us / 1e3,
+                "path": ("decode kernel" if esp.espace_linear_forward_launches(sets[0]["p"], n_tok) == 1
+                         and n_tok <= 32 else "tcgen05")}
+    finally:
+        if own:
+            for s in sets:
+                esp.espace_proj_destroy(s["p"])
+    return sweep
+
+
+def config_rows(esp, peak_tc, peak_hbm):
+    """The other workloads of the benchmark, as side rows: the Llama2-7B MLP over a rank
+    sweep, the GPT3-22B layer at 16,384 tokens, calibration over 1,048,576 tokens at K = 6144
+    and K = 24576, the decode sweep on the other Llama2-7B layers, and the whole Llama2-7B
+    layer at batch 1, sequence 4096."""
+    rows = {}
+    seed = synth.BASE_SEED + 500
+    sweep = {}
+    for name, (K, M) in (("gate_up", (4096, 22016)), ("down", (11008, 4096))):
+        for frac in (0.8, 0.7, 0.6, 0.5):
+            L = int(round(frac * K))
+            sweep[f"{name}_{int(frac * 100)}pct"] = layer_row(esp, K, M, L, 8192, seed, peak_tc)
+    rows["llama2_mlp_rank_sweep"] = sweep
+    gpt = {}
+    for name in ("gpt3_22b_qkv", "gpt3_22b_fc1", "gpt3_22b_fc2"):
+        cfg = synth.CONFIGS[name]
+        gpt[name] = layer_row(esp, cfg["K"], cfg["M"], cfg["L"], cfg["N"], seed, peak_tc)
+    rows["gpt3_22b_layer"] = gpt
+    cal = {}
+    n_total, chunk = 1 << 20, 65536
+    for K in (6144, 24576):
+        Xc = synth.ActivationModel(K, seed=seed).sample_device(chunk, stream="calib_tokens")
+        h = esp.espace_calib_create(K)
+        try:
+            esp.espace_calib_accumulate(h, Xc)
+            esp.espace_calib_reset(h)
+            ms = events_ms(lambda i: esp.espace_calib_accumulate(h, Xc), reps=n_total // chunk, warm=0) * (n_total // chunk)
+            esp.espace_check()
+        finally:
+            esp.espace_calib_destroy(h)
+        del Xc
+        cflops = float(n_total) * K * (K + 1)
+        cal[str(K)] = {"tokens": n_total, "ms": ms, "tflops_symmetric": cflops / ms / 1e9,
+                       "frac_tensor_peak": cflops / ms / 1e9 / peak_tc,
+                       "note": "16 accumulations of one 65,536-token chunk"}
+    rows["calibration_1m_tokens"] = cal
+    for name in ("o", "gate_up", "down"):
+        K, M = synth.DECODE_LAYERS[name]
+        rows[f"decode_sweep_llama2_{name}"] = decode_sweep(esp, K, M, K // 2, seed, peak_hbm)
+    layer = {}
+    for name in ("qkv", "o", "gate_up", "down"):
+        K, M = synth.DECODE_LAYERS[name]
+        layer[name] = layer_row(esp, K, M, K // 2, 4096, seed, peak_tc)
+    layer["total"] = {"espace_ms": sum(v["espace_ms"] for v in layer.values()),
+                      "dense_ms": sum(v["dense_ms"] for v in layer.values())}
+    layer["total"]["speedup"] = layer["total"]["dense_ms"] / layer["total"]["espace_ms"]
+    rows["llama2_layer_prefill_batch1_seq4096"] = layer
     return rows
 
 

@@ -118,6 +118,13 @@ int espace_build_projection(espace_calib_t h, const void* W_dev, int64_t M, int6
 int espace_proj_from_host(int64_t K, int64_t M, int64_t L, const double* P_host,
                           const void* W_dev, void* stream, espace_proj_t* out);
 
+/* Synchronous. Step 4 above for a projection already on the device in bf16: PT_dev is P_b^T
+ * as [L][K] row-major bf16 (the L principal directions as rows, e.g. computed by the caller
+ * on the GPU, as the paper does, Sec. A.1); it is copied into the handle (the caller keeps
+ * its buffer) and W' = P_b^T W is folded on the device. Both pointers 16-byte aligned. */
+int espace_proj_from_device(int64_t K, int64_t M, int64_t L, const void* PT_dev,
+                            const void* W_dev, void* stream, espace_proj_t* out);
+
 /* Shape of a projection: any output pointer may be NULL. */
 int espace_proj_shape(espace_proj_t p, int64_t* K, int64_t* M, int64_t* L);
 

@@ -24,7 +24,7 @@ __all__ = [
     "espace_version", "espace_calib_create", "espace_calib_accumulate",
     "espace_calib_accumulate_normalized", "espace_calib_read", "espace_calib_export",
     "espace_calib_import", "espace_calib_reset", "espace_calib_destroy",
-    "espace_build_projection", "espace_proj_from_host", "espace_proj_shape",
+    "espace_build_projection", "espace_proj_from_host", "espace_proj_from_device", "espace_proj_shape",
     "espace_proj_eigenvalues", "espace_proj_read_P", "espace_proj_read_Wfold",
     "espace_proj_export", "espace_proj_import", "espace_proj_destroy",
     "espace_linear_forward", "espace_linear_forward_path", "espace_linear_forward_noalloc",
@@ -75,6 +75,7 @@ _SIGNATURES = {
     "espace_calib_destroy": (None, [_vp]),
     "espace_build_projection": (ctypes.c_int, [_vp, _vp, _i64, _i64, _vp, ctypes.POINTER(_vp)]),
     "espace_proj_from_host": (ctypes.c_int, [_i64, _i64, _i64, _pd, _vp, _vp, ctypes.POINTER(_vp)]),
+    "espace_proj_from_device": (ctypes.c_int, [_i64, _i64, _i64, _vp, _vp, _vp, ctypes.POINTER(_vp)]),
     "espace_proj_shape": (ctypes.c_int, [_vp, _pi64, _pi64, _pi64]),
     "espace_proj_eigenvalues": (ctypes.c_int, [_vp, _pd]),
     "espace_proj_read_P": (ctypes.c_int, [_vp, _pu16]),
@@ -225,6 +226,15 @@ def espace_proj_from_host(P: np.ndarray, W, stream=None) -> int:
     p = _vp()
     _check(lib.espace_proj_from_host(K, int(W.shape[0]), L, _np_ptr(P, ctypes.c_double),
                                      _dev_ptr(W), _stream(stream), ctypes.byref(p)))
+    return p.value
+
+
+def espace_proj_from_device(PT, W, stream=None) -> int:
+    """PT: device bf16 [L][K] (P_b^T), W: device bf16 [M][K]."""
+    L, K = int(PT.shape[0]), int(PT.shape[1])
+    p = _vp()
+    _check(lib.espace_proj_from_device(K, int(W.shape[0]), L, _dev_ptr(PT), _dev_ptr(W), _stream(stream),
+                                       ctypes.byref(p)))
     return p.value
 
 

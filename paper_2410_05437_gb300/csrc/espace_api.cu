@@ -50,6 +50,17 @@ int fail_cuda(cudaError_t e, const char* what)
         if (_e != cudaSuccess) return fail_cuda(_e, what); \
     } while (0)
 
+// As CUDA_TRY, running `cleanup` before returning the error.
+#define CUDA_TRY_OR(expr, what, cleanup)            \
+    do {                                            \
+        cudaError_t _e = (expr);                    \
+        if (_e != cudaSuccess) {                    \
+            const int _rc = fail_cuda(_e, what);    \
+            cleanup;                                \
+            return _rc;                             \
+        }                                           \
+    } while (0)
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 std::atomic<uint64_t> g_wait_limit_ns{4000000000ull};
@@ -425,6 +436,34 @@ int espace_proj_from_host(int64_t K, int64_t M, int64_t L, const double* P_host,
         espace_proj_destroy(p);
         return rc;
     }
+    *out = p;
+    return ESPACE_OK;
+}
+
+int espace_proj_from_device(int64_t K, int64_t M, int64_t L, const void* PT_dev, const void* W_dev, void* stream,
+                            espace_proj_t* out)
+{
+    if (out == nullptr || PT_dev == nullptr || W_dev == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_proj_from_device: null pointer");
+    *out = nullptr;
+    int rc = check_proj_shape(K, M, L);
+    if (rc != ESPACE_OK) return rc;
+    if (!aligned16(W_dev) || !aligned16(PT_dev))
+        return fail(ESPACE_ERR_ALIGN, "espace_proj_from_device: P^T and W must be 16-byte aligned");
+    espace_proj_s* p = nullptr;
+    rc = proj_create(K, M, L, &p);
+    if (rc != ESPACE_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // rows L .. Lp-1 of the handle's P^T are zero
+    CUDA_TRY_OR(cudaMemcpyAsync(p->PT, PT_dev, sizeof(uint16_t) * L * K, cudaMemcpyDeviceToDevice, st),
+                "espace_proj_from_device: copy P^T", espace_proj_destroy(p));
+    if (p->Lp > L)
+        CUDA_TRY_OR(cudaMemsetAsync(p->PT + L * K, 0, sizeof(uint16_t) * (p->Lp - L) * K, st),
+                    "espace_proj_from_device: clear padding", espace_proj_destroy(p));
+    CUDA_TRY_OR(launch_gemm_tn(W_dev, K, p->PT, K, static_cast<int>(M), static_cast<int>(p->Lp), static_cast<int>(K),
+                               p->WfT, p->Lp, st),
+                "espace_proj_from_device: fold launch", espace_proj_destroy(p));
+    CUDA_TRY_OR(cudaStreamSynchronize(st), "espace_proj_from_device: fold", espace_proj_destroy(p));
     *out = p;
     return ESPACE_OK;
 }

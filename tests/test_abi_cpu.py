@@ -37,6 +37,9 @@ def test_error_codes_without_gpu():
     assert e.value.code == 2
     assert esp.lib.espace_host_eigh(None, 3, None, None, 0) == 1      # ESPACE_ERR_ARG
     assert "null" in esp.lib.espace_last_error().decode()
+    out = ctypes.c_void_p()
+    assert esp.lib.espace_proj_from_device(512, 512, 256, None, None, None, ctypes.byref(out)) == 1
+    assert out.value is None
 
 
 @pytest.mark.parametrize("K", [1, 2, 9, 64, 200])

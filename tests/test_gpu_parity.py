@@ -91,6 +91,32 @@ def test_projection_upload_and_fold(esp):
         esp.espace_proj_destroy(p)
 
 
+def test_projection_from_device_matches_host_path(esp):
+    """A bf16 P^T handed over on the device gives the same handle as the fp64 host path
+    after its rounding: bit-identical P and W', and the same outputs."""
+    K, M, L, N = 520, 264, 100, 40
+    P = synth.random_projection(K, L, seed=11)
+    W = dev(synth.weights(M, K, seed=11))
+    Pb = oracle.bf16_round(P)
+    PT = torch.from_numpy(np.ascontiguousarray(Pb.T)).to(torch.bfloat16).cuda()
+    a = esp.espace_proj_from_host(P, W)
+    b = esp.espace_proj_from_device(PT, W)
+    try:
+        assert np.array_equal(esp.espace_proj_read_P(a), esp.espace_proj_read_P(b))
+        assert np.array_equal(esp.espace_proj_read_Wfold(a), esp.espace_proj_read_Wfold(b))
+        _, X, _ = make_layer(K, M, N, seed=11)
+        Ya = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        Yb = torch.empty_like(Ya)
+        esp.espace_linear_forward(a, dev(X), Ya)
+        esp.espace_linear_forward(b, dev(X), Yb)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        assert torch.equal(Ya.view(torch.int16), Yb.view(torch.int16))
+    finally:
+        esp.espace_proj_destroy(a)
+        esp.espace_proj_destroy(b)
+
+
 # ------------------------------------------------------------------------------ forward (Eq. 3)
 
 FORWARD_CASES = [
