@@ -16,7 +16,9 @@ arrays and chains the steps in the order the paper states them:
 * ``forward``           project then contract: the projected linear layer of Eq. 3;
 * ``dense``             Y = W^T X (Eq. 1);
 * ``reconstruct`` / ``projection_mse``  Eq. 5 and Eq. 6;
-* ``autocorr_normalized_sum``           Cor. 1's input-normalized autocorrelation.
+* ``autocorr_normalized_sum``           Cor. 1's input-normalized autocorrelation;
+* ``go_mse_matrix`` / ``build_projection_go``  Thm. 2: C = C_X C_W + C_W C_X, P its L
+  principal eigenvectors (ordered by |eigenvalue|, as the paper does when C is indefinite).
 
 Layout: tokens are rows (``X`` is ``[N, K]``), ``W`` is ``[M, K]`` as in ``nn.Linear``,
 ``P`` is ``[K, L]``, ``W'`` is ``[L, M]``, ``Z`` is ``[N, L]`` and ``Y`` is ``[N, M]``.
@@ -55,6 +57,7 @@ def _load():
         lib.oracle_contract.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp]
         lib.oracle_dense.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp]
         lib.oracle_reconstruct.argtypes = [_dp, _dp, _i64, _i64, _i64, _dp]
+        lib.oracle_go_combine.argtypes = [_dp, _dp, _i64, _dp]
         lib.oracle_projection_mse.restype = ctypes.c_double
         lib.oracle_projection_mse.argtypes = [_dp, _dp, _i64, _i64, _i64]
         _lib = lib
@@ -202,3 +205,34 @@ def projection_mse(X, P) -> float:
     X, P = _f64(X), _f64(P)
     N, K = X.shape
     return float(_load().oracle_projection_mse(_ptr(X), _ptr(P), N, K, P.shape[1]))
+
+
+def weight_autocorr(W) -> np.ndarray:
+    """``C_W = E[w w^T] = W^T W / M`` over the M rows (weight vectors) of ``W`` ([M, K])."""
+    W = _f64(W)
+    return autocorr_sum(W) / W.shape[0]
+
+
+def go_mse_matrix(CX, W) -> np.ndarray:
+    """Thm. 2: ``C = C_X C_W + C_W C_X`` with ``C_W = W^T W / M`` (weights and activations
+    taken as independent, as the paper does)."""
+    CX = _f64(CX)
+    K = CX.shape[0]
+    CW = weight_autocorr(W)
+    assert CW.shape == (K, K)
+    C = np.zeros((K, K))
+    _load().oracle_go_combine(_ptr(CX), _ptr(_f64(CW)), K, _ptr(C))
+    return C
+
+
+def build_projection_go(S, n: int, W, L: int):
+    """Thm. 2 calibration: ``C = C_X C_W + C_W C_X`` from ``C_X = S / n``; eigenvalues
+    ordered by magnitude (largest first; the paper sorts absolute values when C is not
+    positive definite); ``P`` = the first L eigenvectors (signs normalized), ``P_b`` its
+    bf16 rounding. Returns ``(P, P_b, w, sweeps)`` with ``w`` in that order."""
+    C = go_mse_matrix(_f64(S) / float(n), W)
+    w, V, sweeps = eigh(C)
+    order = np.argsort(-np.abs(w), kind="stable")
+    w, V = w[order], V[:, order]
+    P = normalize_signs(V[:, :L])
+    return P, bf16_round(P), w, sweeps

@@ -20,6 +20,7 @@
  *   oracle_projection_mse    E ||x - x~||^2                             (Sec. 3.2, Eq. 6)
  *   oracle_dense             Y = W^T X                                  (Sec. 2.1, Eq. 1)
  *   oracle_autocorr_normalized_sum  sum_t (x_t/|x_t|)(x_t/|x_t|)^T     (Sec. 3.2, Cor. 1)
+ *   oracle_go_combine        C = C_X C_W + C_W C_X                      (Sec. 3.3, Thm. 2)
  *
  * The OpenMP pragmas only split the outermost token / row loop across host cores; each
  * output element is still summed in the plain order of its definition.
@@ -262,4 +263,22 @@ double oracle_projection_mse(const double* X, const double* P, int64_t N, int64_
         total += err;
     }
     return N > 0 ? total / (double)N : 0.0;
+}
+
+/* Thm. 2 (GO-MSE): C = C_X C_W + C_W C_X for K x K matrices, each entry summed in index
+ * order. With C_X = E[x x^T] and C_W = E[w w^T] of independent x and w this is
+ * E[x x^T w w^T + w w^T x x^T], the matrix whose principal eigenvectors minimize the bound
+ * on the GEMM-output error of Prop. 1. */
+void oracle_go_combine(const double* CX, const double* CW, int64_t K, double* C)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < K; ++i)
+        for (int64_t j = 0; j < K; ++j) {
+            double a = 0.0, b = 0.0;
+            for (int64_t k = 0; k < K; ++k) {
+                a += CX[i * K + k] * CW[k * K + j];
+                b += CW[i * K + k] * CX[k * K + j];
+            }
+            C[i * K + j] = a + b;
+        }
 }

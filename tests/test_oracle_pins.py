@@ -280,3 +280,72 @@ def test_rounded_intermediates_are_bf16_values():
     assert np.array_equal(Z, oracle.bf16_round(Z))
     assert np.array_equal(Wf, oracle.bf16_round(Wf))
     assert np.array_equal(Z, oracle.bf16_round(oracle.project(X, P, round_bf16=False)))
+
+
+# ------------------------------------------------------------------------------ Thm. 2 (GO-MSE)
+
+def test_go_matrix_equals_the_pairwise_expectation():
+    """Thm. 2: E[x x^T w w^T + w w^T x x^T] over independent x (tokens) and w (weight
+    vectors), written out over every (token, weight) pair with plain loops, is
+    C_X C_W + C_W C_X."""
+    r = np.random.default_rng(21)
+    n, M, K = 5, 3, 4
+    X = r.standard_normal((n, K))
+    W = r.standard_normal((M, K))
+    E = [[0.0] * K for _ in range(K)]
+    for t in range(n):
+        for m in range(M):
+            x, w = X[t], W[m]
+            xw = sum(x[k] * w[k] for k in range(K))
+            for i in range(K):
+                for j in range(K):
+                    E[i][j] += x[i] * xw * w[j] + w[i] * xw * x[j]
+    E = np.array(E) / (n * M)
+    C = oracle.go_mse_matrix(oracle.autocorr_sum(X) / n, W)
+    assert np.allclose(C, E, rtol=0, atol=1e-12)
+    assert np.array_equal(C, C.T)
+
+
+def test_go_bound_term_is_half_the_quadratic_form():
+    """The P-dependent term of Prop. 1's GO-MSE bound, E[<w,x> <w,x~>] over all (token,
+    weight) pairs, equals 1/2 sum_i p_i^T C p_i for any orthonormal P -- the identity the
+    proof of Thm. 2 rests on."""
+    r = np.random.default_rng(22)
+    n, M, K, L = 20, 9, 6, 3
+    X = r.standard_normal((n, K)) * np.linspace(2.0, 0.5, K)
+    W = r.standard_normal((M, K))
+    P, _ = np.linalg.qr(r.standard_normal((K, L)))
+    Xt = oracle.reconstruct(X, P)
+    lhs = np.mean([(W[m] @ X[t]) * (W[m] @ Xt[t]) for t in range(n) for m in range(M)])
+    C = oracle.go_mse_matrix(oracle.autocorr_sum(X) / n, W)
+    rhs = 0.5 * np.trace(P.T @ C @ P)
+    assert abs(lhs - rhs) <= 1e-12 * max(1.0, abs(rhs))
+
+
+def test_go_reduces_to_mse_for_isotropic_weights():
+    """Orthogonal weight rows give C_W = I / K, so C = (2/K) C_X: GO-MSE picks Thm. 1's P
+    with eigenvalues scaled by 2/K."""
+    r = np.random.default_rng(23)
+    n, K, L = 60, 8, 3
+    X = r.standard_normal((n, K)) * np.linspace(3.0, 0.2, K)
+    Q, _ = np.linalg.qr(r.standard_normal((K, K)))
+    S = oracle.autocorr_sum(X)
+    P_go, _, w_go, _ = oracle.build_projection_go(S, n, Q, L)
+    P_mse, _, w_mse, _ = oracle.build_projection(S, n, L)
+    assert np.allclose(P_go, P_mse, rtol=0, atol=1e-9)
+    assert np.allclose(w_go, (2.0 / K) * w_mse, rtol=1e-10, atol=1e-14)
+
+
+def test_go_eigenvalues_ordered_by_magnitude():
+    """An indefinite C (this seed has a negative eigenvalue): the order is by |eigenvalue|,
+    as the paper does when C is not positive definite, and C = V diag(w) V^T still holds."""
+    r = np.random.default_rng(0)
+    X = r.standard_normal((50, 6))
+    W = r.standard_normal((7, 6))
+    S = oracle.autocorr_sum(X)
+    C = oracle.go_mse_matrix(S / 50, W)
+    P, _, w, _ = oracle.build_projection_go(S, 50, W, 6)
+    assert (w < 0).any()
+    assert np.all(np.diff(np.abs(w)) <= 1e-15)
+    assert np.allclose(P.T @ P, np.eye(6), atol=1e-12)
+    assert np.allclose(P @ np.diag(w) @ P.T, C, atol=1e-12 * np.abs(w).max())
