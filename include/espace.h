@@ -112,6 +112,17 @@ void espace_calib_destroy(espace_calib_t h);
 int espace_build_projection(espace_calib_t h, const void* W_dev, int64_t M, int64_t L,
                             void* stream, espace_proj_t* out);
 
+/* Synchronous. As espace_build_projection, with Thm. 2's criterion (GO-MSE, Sec. 3.3): P
+ * holds the L principal eigenvectors of C = C_X C_W + C_W C_X, where C_X = S / n is the
+ * handle's autocorrelation (plain, or normalized for the GO-MSE variant with L2
+ * normalization) and C_W = W^T W / M is the autocorrelation of the M weight rows (computed
+ * on the tensor cores), taking weights and activations as independent. C_W is formed and
+ * C_X C_W multiplied in fp64 on the device; C may be indefinite, so eigenvalues (and
+ * espace_proj_eigenvalues) are ordered by magnitude, largest first, as the paper does.
+ * Temporary device memory: 28 K^2 bytes. */
+int espace_build_projection_go(espace_calib_t h, const void* W_dev, int64_t M, int64_t L,
+                               void* stream, espace_proj_t* out);
+
 /* Synchronous. Same as steps 3 (rounding only) and 4 above for a given fp64 P_host
  * ([K][L], row-major), with no eigen-solve: used to feed one projection to several
  * implementations. */

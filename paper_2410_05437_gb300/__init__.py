@@ -24,7 +24,8 @@ __all__ = [
     "espace_version", "espace_calib_create", "espace_calib_accumulate",
     "espace_calib_accumulate_normalized", "espace_calib_read", "espace_calib_export",
     "espace_calib_import", "espace_calib_reset", "espace_calib_destroy",
-    "espace_build_projection", "espace_proj_from_host", "espace_proj_from_device", "espace_proj_shape",
+    "espace_build_projection", "espace_build_projection_go", "espace_proj_from_host", "espace_proj_from_device",
+    "espace_proj_shape",
     "espace_proj_eigenvalues", "espace_proj_read_P", "espace_proj_read_Wfold",
     "espace_proj_export", "espace_proj_import", "espace_proj_destroy",
     "espace_linear_forward", "espace_linear_forward_path", "espace_linear_forward_noalloc",
@@ -76,6 +77,7 @@ _SIGNATURES = {
     "espace_build_projection": (ctypes.c_int, [_vp, _vp, _i64, _i64, _vp, ctypes.POINTER(_vp)]),
     "espace_proj_from_host": (ctypes.c_int, [_i64, _i64, _i64, _pd, _vp, _vp, ctypes.POINTER(_vp)]),
     "espace_proj_from_device": (ctypes.c_int, [_i64, _i64, _i64, _vp, _vp, _vp, ctypes.POINTER(_vp)]),
+    "espace_build_projection_go": (ctypes.c_int, [_vp, _vp, _i64, _i64, _vp, ctypes.POINTER(_vp)]),
     "espace_proj_shape": (ctypes.c_int, [_vp, _pi64, _pi64, _pi64]),
     "espace_proj_eigenvalues": (ctypes.c_int, [_vp, _pd]),
     "espace_proj_read_P": (ctypes.c_int, [_vp, _pu16]),
@@ -217,6 +219,13 @@ def espace_build_projection(h: int, W, L: int, stream=None) -> int:
     p = _vp()
     _check(lib.espace_build_projection(h, _dev_ptr(W), int(W.shape[0]), int(L), _stream(stream),
                                        ctypes.byref(p)))
+    return p.value
+
+
+def espace_build_projection_go(h: int, W, L: int, stream=None) -> int:
+    p = _vp()
+    _check(lib.espace_build_projection_go(h, _dev_ptr(W), int(W.shape[0]), int(L), _stream(stream),
+                                          ctypes.byref(p)))
     return p.value
 
 

@@ -8,6 +8,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <mutex>
 #include <string>
@@ -185,6 +186,20 @@ struct espace_proj_s {
     float* part = nullptr;         // split reductions of the few-token products (fp32)
     int64_t part_cap = 0;
     std::mutex mu;                 // guards scratch growth
+};
+
+// A device allocation freed when it goes out of scope.
+struct DevBuf {
+    void* ptr = nullptr;
+    ~DevBuf()
+    {
+        if (ptr) cudaFree(ptr);
+    }
+    template <typename T>
+    T* as() const
+    {
+        return static_cast<T*>(ptr);
+    }
 };
 
 extern "C" {
@@ -432,6 +447,65 @@ int espace_proj_from_host(int64_t K, int64_t M, int64_t L, const double* P_host,
     rc = proj_create(K, M, L, &p);
     if (rc != ESPACE_OK) return rc;
     rc = proj_upload_and_fold(p, P_host, W_dev, static_cast<cudaStream_t>(stream));
+    if (rc != ESPACE_OK) {
+        espace_proj_destroy(p);
+        return rc;
+    }
+    *out = p;
+    return ESPACE_OK;
+}
+
+int espace_build_projection_go(espace_calib_t h, const void* W_dev, int64_t M, int64_t L, void* stream,
+                               espace_proj_t* out)
+{
+    if (out == nullptr || h == nullptr || W_dev == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_build_projection_go: null pointer");
+    *out = nullptr;
+    const int64_t K = h->K;
+    int rc = check_proj_shape(K, M, L);
+    if (rc != ESPACE_OK) return rc;
+    if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_build_projection_go: W not 16-byte aligned");
+    if (h->n == 0) return fail(ESPACE_ERR_STATE, "espace_build_projection_go: no calibration tokens");
+    DeviceGuard g(h->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t kk = static_cast<size_t>(K * K);
+    DevBuf cw_upper, cx, cw, t;
+    cudaError_t e = cudaMalloc(&cw_upper.ptr, sizeof(float) * kk);
+    if (e == cudaSuccess) e = cudaMalloc(&cx.ptr, sizeof(double) * kk);
+    if (e == cudaSuccess) e = cudaMalloc(&cw.ptr, sizeof(double) * kk);
+    if (e == cudaSuccess) e = cudaMalloc(&t.ptr, sizeof(double) * kk);
+    if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_build_projection_go: %s", cudaGetErrorString(e));
+    // C_W = W^T W / M: the calibration SYRK with the M weight rows as its tokens
+    CUDA_TRY(launch_zero_f32(cw_upper.as<float>(), static_cast<int64_t>(kk), st), "build_projection_go: clear");
+    CUDA_TRY(launch_syrk_upper(W_dev, M, static_cast<int>(K), cw_upper.as<float>(), st), "build_projection_go: C_W");
+    CUDA_TRY(launch_sym_full_f64(h->S, K, 1.0 / static_cast<double>(h->n), cx.as<double>(), st),
+             "build_projection_go: C_X");
+    CUDA_TRY(launch_sym_full_f64(cw_upper.as<float>(), K, 1.0 / static_cast<double>(M), cw.as<double>(), st),
+             "build_projection_go: C_W full");
+    // T = C_X C_W in fp64; C = T + T^T = C_X C_W + C_W C_X (both factors symmetric)
+    CUDA_TRY(launch_gemm_f64(cx.as<double>(), cw.as<double>(), static_cast<int>(K), t.as<double>(), st),
+             "build_projection_go: product");
+    std::vector<double> T(kk), C(kk), w(K), V(kk);
+    CUDA_TRY(cudaStreamSynchronize(st), "build_projection_go: sync");
+    CUDA_TRY(cudaMemcpy(T.data(), t.ptr, sizeof(double) * kk, cudaMemcpyDeviceToHost), "build_projection_go: read");
+    for (int64_t i = 0; i < K; ++i)
+        for (int64_t j = 0; j < K; ++j) C[i * K + j] = T[i * K + j] + T[j * K + i];
+    rc = host_eigh(C.data(), K, w.data(), V.data(), 0);
+    if (rc != ESPACE_OK) return fail(rc, "espace_build_projection_go: eigen-solver did not converge");
+    // C may be indefinite: order by |eigenvalue|, largest first (ties keep the signed order)
+    std::vector<int64_t> order(K);
+    for (int64_t i = 0; i < K; ++i) order[i] = i;
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int64_t a, int64_t b) { return std::fabs(w[a]) > std::fabs(w[b]); });
+    std::vector<double> P(static_cast<size_t>(K * L)), wo(K);
+    for (int64_t i = 0; i < K; ++i) wo[i] = w[order[i]];
+    for (int64_t k = 0; k < K; ++k)
+        for (int64_t l = 0; l < L; ++l) P[k * L + l] = V[k * K + order[l]];
+    espace_proj_s* p = nullptr;
+    rc = proj_create(K, M, L, &p);
+    if (rc != ESPACE_OK) return rc;
+    p->evals = wo;
+    rc = proj_upload_and_fold(p, P.data(), W_dev, st);
     if (rc != ESPACE_OK) {
         espace_proj_destroy(p);
         return rc;

@@ -78,6 +78,11 @@ cudaError_t launch_normalize_rows(const void* X, int64_t N, int K, void* Xn, cud
 // ESPACE_ERR_TIMEOUT in the status word and returns.
 cudaError_t launch_wait_timeout(uint64_t limit_ns, cudaStream_t stream);
 
+// C[K][K] (fp64) = scale * (the symmetric matrix whose upper triangle is Su, fp32).
+cudaError_t launch_sym_full_f64(const float* Su, int64_t K, double scale, double* C, cudaStream_t stream);
+// T = A B for K x K row-major fp64 matrices.
+cudaError_t launch_gemm_f64(const double* A, const double* B, int K, double* T, cudaStream_t stream);
+
 // Fills dst[count] with zeros (fp32).
 cudaError_t launch_zero_f32(float* dst, int64_t count, cudaStream_t stream);
 

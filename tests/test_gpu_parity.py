@@ -374,6 +374,58 @@ def test_build_projection_tiny_config(esp):
         esp.espace_calib_destroy(h)
 
 
+@pytest.mark.parametrize("normalized", [False, True])
+def test_build_projection_go_tiny_config(esp, normalized):
+    """Thm. 2 (GO-MSE, and with Cor. 1's normalized calibration its L2-normalized variant):
+    eigenvalues of C = C_X C_W + C_W C_X and the L-dimensional subspace against the oracle,
+    then the forward with the library's P."""
+    cfg = synth.CONFIGS["tiny"]
+    K, M, L, N, n = cfg["K"], cfg["M"], cfg["L"], cfg["N"], cfg["calib_tokens"]
+    seed = synth.config_seed("tiny")
+    model = synth.ActivationModel(K, seed=seed, outliers=cfg["outliers"], lognormal_sigma=cfg["lognormal_sigma"])
+    Xc = model.sample(n, stream="calib_tokens")
+    X = model.sample(N)
+    W = synth.weights(M, K, seed=seed)
+    h = esp.espace_calib_create(K)
+    p = None
+    try:
+        if normalized:
+            # the library rounds the unit-norm tokens to bf16 before the tensor-core product
+            # (its norms in fp32: an occasional rounding differs, hence the looser tolerance)
+            esp.espace_calib_accumulate_normalized(h, dev(Xc))
+            Xf = f64(Xc)
+            S_o = oracle.autocorr_sum(oracle.bf16_round(Xf / np.linalg.norm(Xf, axis=1, keepdims=True)))
+            tol = 1e-4
+        else:
+            esp.espace_calib_accumulate(h, dev(Xc))
+            S_o = oracle.autocorr_sum(f64(Xc))
+            tol = 1e-5
+        p = esp.espace_build_projection_go(h, dev(W), L)
+        w = esp.espace_proj_eigenvalues(p)
+        P_o, Pb_o, w_o, _ = oracle.build_projection_go(S_o, n, f64(W), L)
+        scale = np.abs(w_o).max()
+        assert np.all(np.diff(np.abs(w)) <= 1e-12 * scale)          # ordered by magnitude
+        assert np.allclose(np.sort(w), np.sort(w_o), rtol=0, atol=tol * scale)
+        Pb = synth.bf16_to_f64(torch.from_numpy(esp.espace_proj_read_P(p).view(np.int16)).view(torch.bfloat16))
+        # same subspace: projector distance within Davis-Kahan (C error / gap at the cut) plus
+        # the bf16 rounding of P
+        gap = abs(w_o[L - 1]) - abs(w_o[L])
+        C_o = oracle.go_mse_matrix(S_o / n, f64(W))
+        dC = tol * np.linalg.norm(C_o)
+        proj = np.linalg.norm(Pb @ Pb.T - P_o @ P_o.T, 2)
+        assert proj <= dC / gap + 2e-2, (proj, dC / gap)
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Y)
+        torch.cuda.synchronize()
+        Y_o, _, _ = oracle.forward(f64(X), Pb, f64(W))
+        assert_y_close(Y, Y_o)
+        esp.espace_check()
+    finally:
+        if p:
+            esp.espace_proj_destroy(p)
+        esp.espace_calib_destroy(h)
+
+
 def test_proj_export_import_roundtrip(esp):
     K, M, L = 256, 128, 96
     P = synth.random_projection(K, L, seed=21)
