@@ -344,6 +344,8 @@ constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 256;
 // tokens) and its epilogue adds the chunks in fp32 registers, so that long token runs do
 // not lose precision in the tensor core's accumulator.
 constexpr int SYRK_CHUNK = 16;
+// Tile rows per group of the grouped tile order of full-grid products.
+constexpr int PAIR_GROUP_M = 8;
 
 template <bool SYRK>
 struct PairShape {
@@ -412,8 +414,15 @@ __device__ __forceinline__ void pair_decode(const PairArgs& a, int item, int& pr
         tm = t.x;
         tn = t.y;
     } else {
-        tm = tile / p.tiles_n;
-        tn = tile - tm * p.tiles_n;
+        // grouped order: PAIR_GROUP_M tile rows at a time, columns outer within the group, so
+        // that the tiles one wave of CTA pairs runs together share A and B slices in L2
+        const int tiles_m = p.num_tiles / p.tiles_n;
+        const int per_group = PAIR_GROUP_M * p.tiles_n;
+        const int first_m = (tile / per_group) * PAIR_GROUP_M;
+        const int group_m = min(tiles_m - first_m, PAIR_GROUP_M);
+        const int in_group = tile - (tile / per_group) * per_group;
+        tm = first_m + in_group % group_m;
+        tn = in_group / group_m;
     }
     kb0 = split * p.kb_per_split;
     kb1 = min(kb0 + p.kb_per_split, p.kblocks);
