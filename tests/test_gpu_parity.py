@@ -143,6 +143,13 @@ FORWARD_CASES = [
     (256, 2048, 1000, 1000, 0),    # 256-token tiles
     (129, 520, 264, 100, 1),       # 256-token tile, ragged
     (7, 1024, 776, 448, 1),        # fewer tokens than one MMA's rows
+    # one token on the decode kernel, across its stage layouts
+    (1, 4096, 12288, 2048, 0),     # Llama2 QKV layer
+    (1, 11008, 4096, 1376, 2),     # K beyond one 2048-wide k-block, ragged
+    (1, 1040, 22016, 600, 0),      # wide M, ragged L, K not a multiple of 64
+    (1, 24, 8, 1, 0),              # rank 1
+    (1, 16384, 264, 128, 0),       # large K, few output rows
+    (1, 24576, 512, 128, 2),       # K of the GPT3-22B FC2 layer
 ]
 
 
@@ -235,6 +242,38 @@ def test_linear_forward_repeated_calls_and_scratch_growth(esp):
             torch.cuda.synchronize()
             Y_o, _, _ = oracle.forward(f64(X), Pb, f64(W), Wf=Wf_o)
             assert_y_close(Y, Y_o)
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+def test_single_token_forward_repeated_and_interleaved(esp):
+    """Successive single tokens, and calls with more tokens in between, each match the
+    oracle (the decode kernel's grid barrier and scratch are left ready for the next call);
+    the same token twice agrees to within one bf16 ulp (partial sums meet in arrival order)."""
+    K, M, L = 4096, 4096, 1024
+    P = synth.random_projection(K, L, seed=8)
+    W = synth.weights(M, K, seed=8)
+    p = esp.espace_proj_from_host(P, dev(W))
+    model = synth.ActivationModel(K, seed=8)
+    Pb = oracle.bf16_round(P)
+    Wf_o = oracle.fold(Pb, f64(W))
+    try:
+        X = model.sample(12, chunk=12)
+        first = None
+        for N, rows in ((1, slice(0, 1)), (1, slice(1, 2)), (8, slice(2, 10)), (1, slice(0, 1)), (1, slice(10, 11))):
+            Xs = X[rows].contiguous()
+            Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+            esp.espace_linear_forward(p, dev(Xs), Y)
+            torch.cuda.synchronize()
+            esp.espace_check()
+            Y_o, _, _ = oracle.forward(f64(Xs), Pb, f64(W), Wf=Wf_o)
+            assert_y_close(Y, Y_o)
+            if rows == slice(0, 1):
+                if first is None:
+                    first = Y.clone()
+                else:
+                    ulp = (first.float() - Y.float()).abs() <= first.float().abs() * 2.0 ** -7
+                    assert bool(ulp.all())
     finally:
         esp.espace_proj_destroy(p)
 
