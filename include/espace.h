@@ -131,7 +131,7 @@ int espace_proj_from_host(int64_t K, int64_t M, int64_t L, const double* P_host,
 
 /* Synchronous. Step 4 above for a projection already on the device in bf16: PT_dev is P_b^T
  * as [L][K] row-major bf16 (the L principal directions as rows, e.g. computed by the caller
- * on the GPU, as the paper does, Sec. A.1); it is copied into the handle (the caller keeps
+ * on the GPU, as the paper does, Sec. B.1); it is copied into the handle (the caller keeps
  * its buffer) and W' = P_b^T W is folded on the device. Both pointers 16-byte aligned. */
 int espace_proj_from_device(int64_t K, int64_t M, int64_t L, const void* PT_dev,
                             const void* W_dev, void* stream, espace_proj_t* out);
@@ -159,12 +159,55 @@ int espace_proj_import(int64_t K, int64_t M, int64_t L, const uint16_t* PT_host,
 void espace_proj_destroy(espace_proj_t p);
 
 /* ---------------------------------------------------------------------------------------
+ * Tensor-parallel layers folded onto one GPU (Sec. B.2, Table 2; latency method of Sec. B.4)
+ *
+ * Under tensor parallelism the paper applies ESPACE per rank, each rank r of tp with its
+ * own projection P_r of L components. Folded onto one GPU the layer computes, for
+ *   ESPACE_TP_COLUMN (column-parallel: QKV, FC1; rank r holds all K inputs and the output
+ *   columns [r M/tp, (r+1) M/tp)):  Y[:, r M/tp ..] = bf16(X P_r) W'_r,  W'_r = P_r^T W_r^T
+ *   with W_r the rank's M/tp rows of W (P_r: K x L);
+ *   ESPACE_TP_ROW (row-parallel: attention projection, FC2; rank r holds the inputs
+ *   [r K/tp, (r+1) K/tp) and all M outputs):  Y = sum_r bf16(X_r P_r) W'_r,
+ *   W'_r = P_r^T W[:, r K/tp ..]^T (P_r: K/tp x L).
+ * Both are two products: one dense and one block-diagonal with one block per rank (the
+ * second for COLUMN, the first for ROW), each a tcgen05 launch on CTA pairs; Z ([N][tp L],
+ * the ranks' intermediates side by side) is rounded to bf16 as in the plain layer.
+ * Shapes: 1 <= tp <= 8; L a multiple of 64 with L <= K / tp (ROW) or L <= K (COLUMN);
+ * COLUMN: M / tp a positive multiple of 8; ROW: K / tp a multiple of 64. The forward
+ * calls (espace_linear_forward, _path with any path, _launches) accept these handles and
+ * always run the two launches; espace_proj_read_P writes the tp bf16 projections as
+ * [tp][Kr][L]; espace_proj_read_Wfold, _export and espace_linear_forward_noalloc return
+ * ESPACE_ERR_STATE for them.
+ * ------------------------------------------------------------------------------------- */
+#define ESPACE_TP_COLUMN 1
+#define ESPACE_TP_ROW    2
+
+/* Synchronous. A tensor-parallel layer from tp given fp64 projections P_host, [tp][Kr][L]
+ * row-major (Kr = K for COLUMN, K / tp for ROW), each rounded to bf16, and W_dev ([M][K]
+ * bf16, read once): the ranks' W'_r are folded on the GPU (fp32 accumulation, bf16). */
+int espace_proj_tp_from_host(int kind, int tp, int64_t K, int64_t M, int64_t L, const double* P_host,
+                             const void* W_dev, void* stream, espace_proj_t* out);
+
+/* Synchronous. As espace_build_projection (Thm. 1 per rank) for a tensor-parallel layer:
+ * rank r's autocorrelation is that of its own inputs, i.e. C = S / n for COLUMN (every rank
+ * sees all K inputs, so the ranks' projections coincide and the returned handle is the
+ * plain layer with the rank's L; the paper's per-rank L, Table 2) and the r-th diagonal
+ * K/tp x K/tp block of C for ROW (tp eigen-solves of size K / tp; the handle's
+ * eigenvalues are the tp ranks' K / tp values, each block decreasing). */
+int espace_build_projection_tp(espace_calib_t h, const void* W_dev, int64_t M, int64_t L, int kind, int tp,
+                               void* stream, espace_proj_t* out);
+
+/* The handle's tensor-parallel kind (0 for a plain layer) and rank count (1 for a plain
+ * layer). Either pointer may be null. */
+int espace_proj_tp_info(espace_proj_t p, int* kind, int* tp);
+
+/* ---------------------------------------------------------------------------------------
  * Forward (Sec. 2.2, Eq. 3)
  * ------------------------------------------------------------------------------------- */
 
 /* Async. Y = (P^T W)^T (P^T X) for the N tokens of X_dev ([N][K] bf16) into Y_dev
  * ([N][M] bf16): Z = X P is accumulated in fp32 and rounded to bf16 (the paper computes in
- * BF16, Sec. A.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 16 runs
+ * BF16, Sec. B.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 16 runs
  * a bandwidth-bound kernel that streams P and W' once; N <= 256 runs two tcgen05 launches
  * with the weights as the 128-row operand (phase 1 splits its reduction over the SMs and
  * adds the fp32 partials in a fixed order, so results are reproducible bit for bit);

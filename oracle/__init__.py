@@ -18,7 +18,9 @@ arrays and chains the steps in the order the paper states them:
 * ``reconstruct`` / ``projection_mse``  Eq. 5 and Eq. 6;
 * ``autocorr_normalized_sum``           Cor. 1's input-normalized autocorrelation;
 * ``go_mse_matrix`` / ``build_projection_go``  Thm. 2: C = C_X C_W + C_W C_X, P its L
-  principal eigenvectors (ordered by |eigenvalue|, as the paper does when C is indefinite).
+  principal eigenvectors (ordered by |eigenvalue|, as the paper does when C is indefinite);
+* ``forward_tp`` / ``build_projection_tp``  ESPACE applied per tensor-parallel rank
+  (Sec. B.2, Table 2), the ranks folded onto one device (Sec. B.4).
 
 Layout: tokens are rows (``X`` is ``[N, K]``), ``W`` is ``[M, K]`` as in ``nn.Linear``,
 ``P`` is ``[K, L]``, ``W'`` is ``[L, M]``, ``Z`` is ``[N, L]`` and ``Y`` is ``[N, M]``.
@@ -236,3 +238,50 @@ def build_projection_go(S, n: int, W, L: int):
     w, V = w[order], V[:, order]
     P = normalize_signs(V[:, :L])
     return P, bf16_round(P), w, sweeps
+
+
+def forward_tp(X, P_blocks, W, kind: str, round_bf16: bool = True) -> np.ndarray:
+    """ESPACE applied per tensor-parallel rank (Sec. B.2, Table 2), the tp ranks' outputs
+    combined on one device (Sec. B.4). ``P_blocks`` is ``[tp, Kr, L]``: rank r's projection.
+
+    ``kind == "column"`` (QKV, FC1): rank r holds all K inputs and the output rows
+    ``W_r = W[r M/tp : (r+1) M/tp]``; its outputs are the layer of Eq. 3 with ``P_r``
+    (``Kr = K``): ``Y[:, r M/tp ..] = forward(X, P_r, W_r)``.
+    ``kind == "row"`` (attention projection, FC2): rank r holds the inputs
+    ``X_r = X[:, r K/tp : (r+1) K/tp]`` and the matching columns of W (``Kr = K / tp``); the
+    ranks' outputs are summed: ``Y = sum_r forward(X_r, P_r, W[:, r K/tp ..])``.
+    Returns ``Y`` ([N, M], fp64)."""
+    X, W, P_blocks = _f64(X), _f64(W), _f64(P_blocks)
+    N, K = X.shape
+    M = W.shape[0]
+    tp = P_blocks.shape[0]
+    Y = np.zeros((N, M))
+    if kind == "column":
+        assert M % tp == 0 and P_blocks.shape[1] == K
+        Mr = M // tp
+        for r in range(tp):
+            Y[:, r * Mr:(r + 1) * Mr] = forward(X, P_blocks[r], W[r * Mr:(r + 1) * Mr], round_bf16=round_bf16)[0]
+    elif kind == "row":
+        assert K % tp == 0 and P_blocks.shape[1] == K // tp
+        Kr = K // tp
+        for r in range(tp):
+            Y += forward(X[:, r * Kr:(r + 1) * Kr], P_blocks[r], W[:, r * Kr:(r + 1) * Kr], round_bf16=round_bf16)[0]
+    else:
+        raise ValueError(kind)
+    return Y
+
+
+def build_projection_tp(S, n: int, L: int, kind: str, tp: int):
+    """Thm. 1 per tensor-parallel rank: rank r's autocorrelation is that of its own inputs,
+    all of ``C = S / n`` for ``"column"`` (every rank sees all K inputs) and the r-th
+    diagonal ``K/tp x K/tp`` block of C for ``"row"``. Returns ``(P, P_b, w)``: ``[tp, Kr,
+    L]`` fp64 projections, their bf16 rounding, and ``[tp, Kr]`` eigenvalues (decreasing)."""
+    S = _f64(S)
+    K = S.shape[0]
+    Kr = K if kind == "column" else K // tp
+    P = np.zeros((tp, Kr, L))
+    w = np.zeros((tp, Kr))
+    for r in range(tp):
+        Sr = S if kind == "column" else S[r * Kr:(r + 1) * Kr, r * Kr:(r + 1) * Kr]
+        P[r], _, w[r], _ = build_projection(Sr, n, L)
+    return P, bf16_round(P), w

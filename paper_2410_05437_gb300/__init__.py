@@ -33,10 +33,12 @@ __all__ = [
     "espace_check", "espace_debug_wait_timeout", "espace_set_wait_limit_ns", "espace_set_phase_event",
     "espace_host_eigh",
     "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "PATH_TENSOR_SPLIT", "EXPORTED_SYMBOLS",
+    "TP_COLUMN", "TP_ROW", "espace_proj_tp_from_host", "espace_build_projection_tp", "espace_proj_tp_info",
     "espace_linear_forward_launches",
 ]
 
 PATH_AUTO, PATH_TENSOR, PATH_SMALL_N, PATH_TENSOR_SPLIT = 0, 1, 2, 3
+TP_COLUMN, TP_ROW = 1, 2
 
 ERROR_NAMES = {1: "ARG", 2: "SHAPE", 3: "ALIGN", 4: "CUDA", 5: "TIMEOUT", 6: "STATE",
                7: "NOMEM", 8: "NUMERIC"}
@@ -78,6 +80,11 @@ _SIGNATURES = {
     "espace_proj_from_host": (ctypes.c_int, [_i64, _i64, _i64, _pd, _vp, _vp, ctypes.POINTER(_vp)]),
     "espace_proj_from_device": (ctypes.c_int, [_i64, _i64, _i64, _vp, _vp, _vp, ctypes.POINTER(_vp)]),
     "espace_build_projection_go": (ctypes.c_int, [_vp, _vp, _i64, _i64, _vp, ctypes.POINTER(_vp)]),
+    "espace_proj_tp_from_host": (ctypes.c_int, [ctypes.c_int, ctypes.c_int, _i64, _i64, _i64, _pd, _vp, _vp,
+                                                ctypes.POINTER(_vp)]),
+    "espace_build_projection_tp": (ctypes.c_int, [_vp, _vp, _i64, _i64, ctypes.c_int, ctypes.c_int, _vp,
+                                                  ctypes.POINTER(_vp)]),
+    "espace_proj_tp_info": (ctypes.c_int, [_vp, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_int)]),
     "espace_proj_shape": (ctypes.c_int, [_vp, _pi64, _pi64, _pi64]),
     "espace_proj_eigenvalues": (ctypes.c_int, [_vp, _pd]),
     "espace_proj_read_P": (ctypes.c_int, [_vp, _pu16]),
@@ -238,6 +245,32 @@ def espace_proj_from_host(P: np.ndarray, W, stream=None) -> int:
     return p.value
 
 
+def espace_proj_tp_from_host(kind: int, P: np.ndarray, W, stream=None) -> int:
+    """P: fp64 [tp][Kr][L], one projection per tensor-parallel rank (Kr = K for TP_COLUMN,
+    K / tp for TP_ROW); W: device bf16 [M][K]."""
+    P = np.ascontiguousarray(P, dtype=np.float64)
+    tp, Kr, L = P.shape
+    K = int(W.shape[1])
+    p = _vp()
+    _check(lib.espace_proj_tp_from_host(int(kind), int(tp), K, int(W.shape[0]), int(L), _np_ptr(P, ctypes.c_double),
+                                        _dev_ptr(W), _stream(stream), ctypes.byref(p)))
+    return p.value
+
+
+def espace_build_projection_tp(h: int, W, L: int, kind: int, tp: int, stream=None) -> int:
+    p = _vp()
+    _check(lib.espace_build_projection_tp(h, _dev_ptr(W), int(W.shape[0]), int(L), int(kind), int(tp),
+                                          _stream(stream), ctypes.byref(p)))
+    return p.value
+
+
+def espace_proj_tp_info(p: int):
+    """(kind, tp): 0 and 1 for a plain layer."""
+    kind, tp = ctypes.c_int(), ctypes.c_int()
+    _check(lib.espace_proj_tp_info(p, ctypes.byref(kind), ctypes.byref(tp)))
+    return kind.value, tp.value
+
+
 def espace_proj_from_device(PT, W, stream=None) -> int:
     """PT: device bf16 [L][K] (P_b^T), W: device bf16 [M][K]."""
     L, K = int(PT.shape[0]), int(PT.shape[1])
@@ -261,9 +294,12 @@ def espace_proj_eigenvalues(p: int) -> np.ndarray:
 
 
 def espace_proj_read_P(p: int) -> np.ndarray:
-    """P as raw bf16 bits, ``uint16 [K, L]``."""
+    """P as raw bf16 bits, ``uint16 [K, L]``; for a tensor-parallel layer the ranks'
+    projections, ``uint16 [tp, Kr, L]`` (Kr = K, or K / tp for TP_ROW)."""
     K, _, L = espace_proj_shape(p)
-    out = np.zeros((K, L), dtype=np.uint16)
+    kind, tp = espace_proj_tp_info(p)
+    shape = (K, L) if kind == 0 else (tp, K // tp if kind == TP_ROW else K, L)
+    out = np.zeros(shape, dtype=np.uint16)
     _check(lib.espace_proj_read_P(p, _np_ptr(out, ctypes.c_uint16)))
     return out
 

@@ -185,6 +185,11 @@ struct espace_proj_s {
     int* ready = nullptr;          // fused forward: 2 x ceil(zcap / 256) zeroed counters
     float* part = nullptr;         // split reductions of the few-token products (fp32)
     int64_t part_cap = 0;
+    // tensor-parallel layer (tp_kind != 0): Lp = tp * L is the width of Z. COLUMN: PT is
+    // [tp L][K] (rank r's P_r^T in rows r L ..), WfT is [M][L] (rank r's W'_r^T in rows
+    // r M/tp ..). ROW: PT is [tp L][K/tp], WfT is [M][tp L] (rank r's in columns r L ..).
+    int tp = 1;
+    int tp_kind = 0;
     std::mutex mu;                 // guards scratch growth
 };
 
@@ -577,6 +582,140 @@ int espace_build_projection(espace_calib_t h, const void* W_dev, int64_t M, int6
     return ESPACE_OK;
 }
 
+// ---------------------------------------------------------------------------- tensor parallel
+
+static int check_tp_shape(int kind, int tp, int64_t K, int64_t M, int64_t L)
+{
+    if (kind != ESPACE_TP_COLUMN && kind != ESPACE_TP_ROW) return fail(ESPACE_ERR_ARG, "tensor parallel: unknown kind %d", kind);
+    if (tp < 1 || tp > 8) return fail(ESPACE_ERR_SHAPE, "tensor parallel: tp=%d must be in [1, 8]", tp);
+    if (K < 8 || K % 8 != 0 || K > 65536) return fail(ESPACE_ERR_SHAPE, "tensor parallel: K=%lld", (long long)K);
+    if (M < 8 || M % 8 != 0 || M > (int64_t(1) << 30)) return fail(ESPACE_ERR_SHAPE, "tensor parallel: M=%lld", (long long)M);
+    if (L < 64 || L % 64 != 0) return fail(ESPACE_ERR_SHAPE, "tensor parallel: L=%lld must be a positive multiple of 64", (long long)L);
+    if (kind == ESPACE_TP_COLUMN) {
+        if (M % tp != 0 || (M / tp) % 8 != 0)
+            return fail(ESPACE_ERR_SHAPE, "tensor parallel: M/tp must be a multiple of 8 (M=%lld, tp=%d)", (long long)M, tp);
+        if (L > K) return fail(ESPACE_ERR_SHAPE, "tensor parallel: L=%lld > K=%lld", (long long)L, (long long)K);
+    } else {
+        if (K % tp != 0 || (K / tp) % 64 != 0)
+            return fail(ESPACE_ERR_SHAPE, "tensor parallel: K/tp must be a multiple of 64 (K=%lld, tp=%d)", (long long)K, tp);
+        if (L > K / tp) return fail(ESPACE_ERR_SHAPE, "tensor parallel: L=%lld > K/tp=%lld", (long long)L, (long long)(K / tp));
+    }
+    return ESPACE_OK;
+}
+
+// Allocates a tensor-parallel handle, uploads the tp projections (fp64 [tp][Kr][L]) as bf16
+// P^T blocks and folds each rank's W'_r on the GPU.
+static int tp_create_and_fold(int kind, int tp, int64_t K, int64_t M, int64_t L, const double* P, const void* W,
+                              cudaStream_t st, espace_proj_s** out)
+{
+    DeviceInfo* dev = nullptr;
+    int rc = device_info(&dev);
+    if (rc != ESPACE_OK) return rc;
+    const int64_t Kr = kind == ESPACE_TP_COLUMN ? K : K / tp, Mr = kind == ESPACE_TP_COLUMN ? M / tp : M;
+    espace_proj_s* p = new espace_proj_s();
+    p->K = K;
+    p->M = M;
+    p->L = L;
+    p->Lp = tp * L;
+    p->tp = tp;
+    p->tp_kind = kind;
+    p->device = dev->device;
+    cudaError_t e = cudaMalloc(&p->PT, sizeof(uint16_t) * tp * L * Kr);
+    if (e == cudaSuccess) e = cudaMalloc(&p->WfT, sizeof(uint16_t) * M * (kind == ESPACE_TP_COLUMN ? L : tp * L));
+    if (e == cudaSuccess) e = cudaMalloc(&p->bar, 64);
+    if (e == cudaSuccess) e = cudaMemset(p->bar, 0, 64);
+    if (e != cudaSuccess) {
+        espace_proj_destroy(p);
+        return fail(ESPACE_ERR_NOMEM, "tensor parallel: cudaMalloc: %s", cudaGetErrorString(e));
+    }
+    std::vector<uint16_t> pt(static_cast<size_t>(tp * L * Kr));
+    for (int r = 0; r < tp; ++r)
+        for (int64_t l = 0; l < L; ++l)
+            for (int64_t k = 0; k < Kr; ++k)
+                pt[(r * L + l) * Kr + k] = bf16_from_double(P[(r * Kr + k) * L + l]);
+    CUDA_TRY_OR(cudaStreamSynchronize(st), "tensor parallel: sync", espace_proj_destroy(p));
+    CUDA_TRY_OR(cudaMemcpy(p->PT, pt.data(), sizeof(uint16_t) * pt.size(), cudaMemcpyHostToDevice),
+                "tensor parallel: upload P", espace_proj_destroy(p));
+    const uint16_t* Wb = static_cast<const uint16_t*>(W);
+    for (int r = 0; r < tp; ++r) {
+        cudaError_t f;
+        if (kind == ESPACE_TP_COLUMN)   // W'_r^T [M/tp][L] = W_r [M/tp][K] P_r
+            f = launch_gemm_tn(Wb + r * Mr * K, K, p->PT + r * L * K, K, static_cast<int>(Mr), static_cast<int>(L),
+                               static_cast<int>(K), p->WfT + r * Mr * L, L, st);
+        else                            // W'_r^T [M][L] = W[:, r K/tp ..] P_r, columns r L .. of WfT
+            f = launch_gemm_tn(Wb + r * Kr, K, p->PT + r * L * Kr, Kr, static_cast<int>(M), static_cast<int>(L),
+                               static_cast<int>(Kr), p->WfT + r * L, tp * L, st);
+        CUDA_TRY_OR(f, "tensor parallel: fold launch", espace_proj_destroy(p));
+    }
+    CUDA_TRY_OR(cudaStreamSynchronize(st), "tensor parallel: fold", espace_proj_destroy(p));
+    *out = p;
+    return ESPACE_OK;
+}
+
+int espace_proj_tp_from_host(int kind, int tp, int64_t K, int64_t M, int64_t L, const double* P_host,
+                             const void* W_dev, void* stream, espace_proj_t* out)
+{
+    if (out == nullptr || P_host == nullptr || W_dev == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_proj_tp_from_host: null pointer");
+    *out = nullptr;
+    int rc = check_tp_shape(kind, tp, K, M, L);
+    if (rc != ESPACE_OK) return rc;
+    if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_proj_tp_from_host: W not 16-byte aligned");
+    espace_proj_s* p = nullptr;
+    rc = tp_create_and_fold(kind, tp, K, M, L, P_host, W_dev, static_cast<cudaStream_t>(stream), &p);
+    if (rc != ESPACE_OK) return rc;
+    *out = p;
+    return ESPACE_OK;
+}
+
+int espace_build_projection_tp(espace_calib_t h, const void* W_dev, int64_t M, int64_t L, int kind, int tp,
+                               void* stream, espace_proj_t* out)
+{
+    if (out == nullptr || h == nullptr || W_dev == nullptr)
+        return fail(ESPACE_ERR_ARG, "espace_build_projection_tp: null pointer");
+    *out = nullptr;
+    const int64_t K = h->K;
+    int rc = check_tp_shape(kind, tp, K, M, L);
+    if (rc != ESPACE_OK) return rc;
+    // every column-parallel rank sees all K inputs: one eigen-solve, the plain layer
+    if (kind == ESPACE_TP_COLUMN) return espace_build_projection(h, W_dev, M, L, stream, out);
+    if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_build_projection_tp: W not 16-byte aligned");
+    if (h->n == 0) return fail(ESPACE_ERR_STATE, "espace_build_projection_tp: no calibration tokens");
+    DeviceGuard g(h->device);
+    std::vector<float> S;
+    rc = read_sum(h, S, stream);
+    if (rc != ESPACE_OK) return rc;
+    std::vector<double> C(static_cast<size_t>(K * K));
+    mirror_scaled(S, K, 1.0 / static_cast<double>(h->n), C.data());
+    const int64_t Kr = K / tp;
+    std::vector<double> P(static_cast<size_t>(tp * Kr * L)), evals(static_cast<size_t>(K));
+    std::vector<double> Cr(static_cast<size_t>(Kr * Kr)), w(Kr), V(static_cast<size_t>(Kr * Kr));
+    for (int r = 0; r < tp; ++r) {
+        // rank r's inputs are features r Kr .. (r+1) Kr: its autocorrelation is C's diagonal block
+        for (int64_t i = 0; i < Kr; ++i)
+            for (int64_t j = 0; j < Kr; ++j) Cr[i * Kr + j] = C[(r * Kr + i) * K + r * Kr + j];
+        rc = host_eigh(Cr.data(), Kr, w.data(), V.data(), 0);
+        if (rc != ESPACE_OK) return fail(rc, "espace_build_projection_tp: eigen-solver did not converge");
+        for (int64_t k = 0; k < Kr; ++k)
+            for (int64_t l = 0; l < L; ++l) P[(r * Kr + k) * L + l] = V[k * Kr + l];
+        for (int64_t i = 0; i < Kr; ++i) evals[r * Kr + i] = w[i];
+    }
+    espace_proj_s* p = nullptr;
+    rc = tp_create_and_fold(kind, tp, K, M, L, P.data(), W_dev, static_cast<cudaStream_t>(stream), &p);
+    if (rc != ESPACE_OK) return rc;
+    p->evals = evals;
+    *out = p;
+    return ESPACE_OK;
+}
+
+int espace_proj_tp_info(espace_proj_t p, int* kind, int* tp)
+{
+    if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_tp_info: null handle");
+    if (kind) *kind = p->tp_kind;
+    if (tp) *tp = p->tp;
+    return ESPACE_OK;
+}
+
 int espace_proj_shape(espace_proj_t p, int64_t* K, int64_t* M, int64_t* L)
 {
     if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_shape: null handle");
@@ -598,17 +737,23 @@ int espace_proj_read_P(espace_proj_t p, uint16_t* P_host)
 {
     if (p == nullptr || P_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_read_P: null pointer");
     DeviceGuard g(p->device);
-    std::vector<uint16_t> pt(static_cast<size_t>(p->Lp * p->K));
+    // plain: P^T is [Lp][K]; tensor parallel: tp blocks of L rows of Kr (K or K / tp)
+    const int64_t nb = p->tp_kind != 0 ? p->tp : 1;
+    const int64_t Kr = p->tp_kind == ESPACE_TP_ROW ? p->K / p->tp : p->K;
+    const int64_t rows = p->tp_kind != 0 ? p->tp * p->L : p->Lp;
+    std::vector<uint16_t> pt(static_cast<size_t>(rows * Kr));
     CUDA_TRY(cudaDeviceSynchronize(), "read_P: sync");
     CUDA_TRY(cudaMemcpy(pt.data(), p->PT, sizeof(uint16_t) * pt.size(), cudaMemcpyDeviceToHost), "read_P: copy");
-    for (int64_t k = 0; k < p->K; ++k)
-        for (int64_t l = 0; l < p->L; ++l) P_host[k * p->L + l] = pt[l * p->K + k];
+    for (int64_t b = 0; b < nb; ++b)
+        for (int64_t k = 0; k < Kr; ++k)
+            for (int64_t l = 0; l < p->L; ++l) P_host[(b * Kr + k) * p->L + l] = pt[(b * p->L + l) * Kr + k];
     return ESPACE_OK;
 }
 
 int espace_proj_read_Wfold(espace_proj_t p, uint16_t* Wf_host)
 {
     if (p == nullptr || Wf_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_read_Wfold: null pointer");
+    if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "espace_proj_read_Wfold: tensor-parallel handle");
     DeviceGuard g(p->device);
     std::vector<uint16_t> wt(static_cast<size_t>(p->M * p->Lp));
     CUDA_TRY(cudaDeviceSynchronize(), "read_Wfold: sync");
@@ -622,6 +767,7 @@ int espace_proj_export(espace_proj_t p, uint16_t* PT_host, uint16_t* WfT_host, d
 {
     if (p == nullptr || PT_host == nullptr || WfT_host == nullptr)
         return fail(ESPACE_ERR_ARG, "espace_proj_export: null pointer");
+    if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "espace_proj_export: tensor-parallel handle");
     DeviceGuard g(p->device);
     CUDA_TRY(cudaDeviceSynchronize(), "proj_export: sync");
     CUDA_TRY(cudaMemcpy(PT_host, p->PT, sizeof(uint16_t) * p->Lp * p->K, cudaMemcpyDeviceToHost), "proj_export: P");
@@ -716,6 +862,40 @@ static int ensure_swap(espace_proj_s* p, int n, int num_sms, cudaStream_t st)
     return ESPACE_OK;
 }
 
+// Tensor-parallel layer: a dense product and a block-diagonal one (one block per rank), Z
+// ([N][tp L]) through the scratch buffer.
+static int tp_forward(espace_proj_s* p, const void* X, int n, void* Y, cudaStream_t st)
+{
+    DeviceGuard g(p->device);
+    int rc = ensure_z(p, n, st);
+    if (rc != ESPACE_OK) return rc;
+    const int tp = p->tp, K = static_cast<int>(p->K), M = static_cast<int>(p->M), L = static_cast<int>(p->L);
+    const int zw = tp * L;   // width of Z
+    int ak0[8], c0[8], cw[8];
+    cudaEvent_t mid = g_phase_event;
+    g_phase_event = nullptr;
+    if (p->tp_kind == ESPACE_TP_COLUMN) {
+        CUDA_TRY(launch_gemm_tn(X, K, p->PT, K, n, zw, K, p->Z, zw, st), "tensor parallel: phase 1");
+        if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+        for (int r = 0; r < tp; ++r) {
+            ak0[r] = r * L;
+            c0[r] = r * (M / tp);
+            cw[r] = M / tp;
+        }
+        CUDA_TRY(launch_gemm_tn_blocks(p->Z, zw, zw, p->WfT, n, tp, ak0, c0, cw, L, Y, M, st), "tensor parallel: phase 2");
+    } else {
+        for (int r = 0; r < tp; ++r) {
+            ak0[r] = r * (K / tp);
+            c0[r] = r * L;
+            cw[r] = L;
+        }
+        CUDA_TRY(launch_gemm_tn_blocks(X, K, K, p->PT, n, tp, ak0, c0, cw, K / tp, p->Z, zw, st), "tensor parallel: phase 1");
+        if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+        CUDA_TRY(launch_gemm_tn(p->Z, zw, p->WfT, zw, n, M, zw, Y, M, st), "tensor parallel: phase 2");
+    }
+    return ESPACE_OK;
+}
+
 // Tokens served by the swapped tcgen05 products (between the decode kernel and the fused
 // CTA-pair launch).
 static bool swap_forward_applies(int n, int path) { return n <= SWAP_MAX_TOKENS && path != ESPACE_PATH_TENSOR_SPLIT; }
@@ -732,6 +912,7 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
     if (path < 0 || path > 3) return fail(ESPACE_ERR_ARG, "espace_linear_forward: unknown path %d", path);
     const int K = static_cast<int>(p->K), M = static_cast<int>(p->M), Lp = static_cast<int>(p->Lp);
     const int n = static_cast<int>(N);
+    if (p->tp_kind != 0) return tp_forward(p, X_dev, n, Y_dev, static_cast<cudaStream_t>(stream));
     DeviceInfo* dev = nullptr;
     {
         DeviceGuard g0(p->device);
@@ -783,6 +964,7 @@ int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path)
         DeviceGuard g(p->device);
         if (device_info(&dev) != ESPACE_OK) return -1;
     }
+    if (p->tp_kind != 0) return 2;
     const int n = static_cast<int>(N), K = static_cast<int>(p->K), M = static_cast<int>(p->M),
               Lp = static_cast<int>(p->Lp);
     const bool small_ok = N <= DECODE_MAX_TOKENS && decode_supported(n, K, Lp, M, dev->num_sms);
@@ -877,6 +1059,7 @@ struct ProjView {
 int proj_view(espace_proj_t p, ProjView* out)
 {
     if (p == nullptr || out == nullptr) return fail(ESPACE_ERR_ARG, "proj_view: null pointer");
+    if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "espace_linear_forward_noalloc: tensor-parallel handle");
     out->K = p->K;
     out->M = p->M;
     out->L = p->L;

@@ -48,6 +48,16 @@ constexpr int SWAP_MAX_TOKENS = 256;
 // Whether the CTA-pair kernels are enabled (ESPACE_DISABLE_PAIR_GEMM=1 turns them off).
 bool pair_kernel_enabled();
 
+// Block-diagonal product on CTA pairs (tensor-parallel ranks folded onto one GPU): output
+// column block g, C[:, c0[g] .. c0[g] + cw[g]) (bf16, leading dimension ldc), is
+// A[:, ak0[g] .. ak0[g] + kdim) (A: rows x a_cols bf16, leading dimension lda) times
+// B[c0[g] .. c0[g] + cw[g])[0 .. kdim) transposed (B: [sum cw][kdim] bf16, rows contiguous).
+// The blocks tile the columns in order (c0[0] = 0, c0[g + 1] = c0[g] + cw[g]); at most 8
+// blocks; kdim and every ak0 are multiples of 64.
+cudaError_t launch_gemm_tn_blocks(const void* A, int64_t lda, int a_cols, const void* B, int rows, int nblocks,
+                                  const int* ak0, const int* c0, const int* cw, int kdim, void* C, int64_t ldc,
+                                  cudaStream_t stream);
+
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
 

@@ -346,6 +346,8 @@ constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 256;
 constexpr int SYRK_CHUNK = 16;
 // Tile rows per group of the grouped tile order of full-grid products.
 constexpr int PAIR_GROUP_M = 8;
+// Diagonal blocks of a block-diagonal product (one per tensor-parallel rank).
+constexpr int PAIR_MAX_BLOCKS = 8;
 
 template <bool SYRK>
 struct PairShape {
@@ -371,6 +373,13 @@ struct PairProblem {
 // (target 8 x tiles_n of product 0: four warps in each of two CTAs per tile);
 // done[tm] counts the second product's producers that passed the check, and the last one
 // resets both, so the counters are zero again for the next launch.
+//
+// Block-diagonal product (problem 0 of a one-product program, nblocks > 0): output column
+// block g, columns [c0[g], c0[g] + cw[g]), is A[:, ak0[g] .. ak0[g] + kdim) times rows
+// [c0[g], c0[g] + cw[g]) of B [total cols][kdim] transposed; its column tiles are
+// tile0[g] .. tile0[g + 1] - 1 of the tile grid. kdim is a multiple of the 64-deep k-block,
+// so a block never reads another block's A columns; B rows of a tile past its block's end
+// belong to the next block and only feed columns that are not stored.
 struct PairArgs {
     PairProblem p[2];
     int nprob;
@@ -378,7 +387,44 @@ struct PairArgs {
     int* done;
     int* status;
     uint64_t wait_limit_ns;
+    int nblocks;
+    int tile0[PAIR_MAX_BLOCKS + 1];
+    int ak0[PAIR_MAX_BLOCKS];
+    int c0[PAIR_MAX_BLOCKS];
+    int cw[PAIR_MAX_BLOCKS];
 };
+
+// Column tile tn of problem prob -> A's k offset, B's first row, the first output column
+// and the end of the output columns that tile may store. Unrolled selects keep the block
+// table out of local memory.
+__device__ __forceinline__ void pair_block_of(const PairArgs& a, int prob, int tn, int cols, int& ak0,
+                                              int& brow, int& ccol, int& cend)
+{
+    if (prob != 0 || a.nblocks == 0) {
+        ak0 = 0;
+        brow = tn * PAIR_BN;
+        ccol = tn * PAIR_BN;
+        cend = cols;
+        return;
+    }
+    int g = 0;
+#pragma unroll
+    for (int i = 1; i < PAIR_MAX_BLOCKS; ++i)
+        if (i < a.nblocks && tn >= a.tile0[i]) g = i;
+    int t0 = 0, k0 = 0, c0 = 0, cw = 0;
+#pragma unroll
+    for (int i = 0; i < PAIR_MAX_BLOCKS; ++i)
+        if (i == g) {
+            t0 = a.tile0[i];
+            k0 = a.ak0[i];
+            c0 = a.c0[i];
+            cw = a.cw[i];
+        }
+    ak0 = k0;
+    brow = c0 + (tn - t0) * PAIR_BN;
+    ccol = brow;
+    cend = c0 + cw;
+}
 
 // Field-wise selection keeps the problem in registers (a dynamic index into the kernel
 // parameters would go through local memory).
@@ -542,8 +588,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                         atomicExch(args.done + tm, 0);
                     }
                 }
+                int ak0, brow, ccol, cend;
+                pair_block_of(args, prob, tn, 0, ak0, brow, ccol, cend);
                 const int row_a = tm * PAIR_BM + static_cast<int>(rank) * 128;
-                const int row_b = tn * PAIR_BN + static_cast<int>(rank) * 128;
+                const int row_b = brow + static_cast<int>(rank) * 128;
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
@@ -561,7 +609,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                         tma_load_2d_pair(sb, mb, bar, row_b, kb * BK);
                         tma_load_2d_pair(sb + 8192, mb, bar, row_b + 64, kb * BK);
                     } else {
-                        tma_load_2d_pair(sa, ma, bar, kb * BK, row_a);
+                        tma_load_2d_pair(sa, ma, bar, ak0 + kb * BK, row_a);
                         tma_load_2d_pair(sb, mb, bar, kb * BK, row_b);
                     }
                     if (++stage == PAIR_STAGES) {
@@ -710,17 +758,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
             const int row = tm * PAIR_BM + row_in_tile;
             const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                    static_cast<uint32_t>(acc * PAIR_BN);
+            int ak0, brow, ccol, cend;
+            pair_block_of(args, prob, tn, pb.cols, ak0, brow, ccol, cend);
 #pragma unroll 1
             for (int c = 0; c < PAIR_BN; c += 32) {
-                const int col0 = tn * PAIR_BN + c;
-                if (col0 >= pb.cols) break;          // uniform across the warp
+                const int col0 = ccol + c;
+                if (col0 >= cend) break;             // uniform across the warp
                 uint32_t v[32];
                 tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
                 tmem_ld_wait();
                 if (row >= pb.rows) continue;
                 __nv_bfloat16* out_row =
                     reinterpret_cast<__nv_bfloat16*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
-                if (col0 + 32 <= pb.cols) {
+                if (col0 + 32 <= cend) {
                     uint4* dst = reinterpret_cast<uint4*>(out_row + col0);
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
@@ -734,7 +784,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                 } else {
 #pragma unroll
                     for (int i = 0; i < 32; ++i)
-                        if (col0 + i < pb.cols)
+                        if (col0 + i < cend)
                             out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
                 }
             }
@@ -878,6 +928,43 @@ cudaError_t launch_gemm_tn_pair(const void* A, int64_t lda, const void* B, int64
 }
 
 }  // namespace
+
+cudaError_t launch_gemm_tn_blocks(const void* A, int64_t lda, int a_cols, const void* B, int rows, int nblocks,
+                                  const int* ak0, const int* c0, const int* cw, int kdim, void* C, int64_t ldc,
+                                  cudaStream_t stream)
+{
+    if (rows <= 0) return cudaSuccess;
+    if (nblocks < 1 || nblocks > PAIR_MAX_BLOCKS || kdim <= 0 || kdim % BK != 0) return cudaErrorInvalidValue;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    if (dev->num_sms < 2) return cudaErrorInvalidConfiguration;
+    PairArgs a{};
+    int cols = 0, tiles = 0;
+    for (int g = 0; g < nblocks; ++g) {
+        if (cw[g] <= 0 || c0[g] != cols || ak0[g] < 0 || ak0[g] % BK != 0 || ak0[g] + kdim > a_cols)
+            return cudaErrorInvalidValue;
+        a.tile0[g] = tiles;
+        a.ak0[g] = ak0[g];
+        a.c0[g] = c0[g];
+        a.cw[g] = cw[g];
+        tiles += (cw[g] + PAIR_BN - 1) / PAIR_BN;
+        cols += cw[g];
+    }
+    a.tile0[nblocks] = tiles;
+    a.nblocks = nblocks;
+    CUtensorMap maps[4];
+    if (!encode_map(&maps[0], A, a_cols, rows, lda, BK, 128)) return cudaErrorInvalidValue;
+    if (!encode_map(&maps[1], B, kdim, cols, kdim, BK, 128)) return cudaErrorInvalidValue;
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+    a.p[0] = pair_problem(rows, cols, kdim, C, ldc);
+    a.p[0].tiles_n = tiles;
+    a.p[0].num_tiles = ((rows + PAIR_BM - 1) / PAIR_BM) * tiles;
+    a.nprob = 1;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return launch_pair<false>(maps, a, dev, stream);
+}
 
 // The CTA-pair kernel is used unless ESPACE_DISABLE_PAIR_GEMM=1 is set in the environment.
 bool pair_kernel_enabled()

@@ -40,6 +40,18 @@ def test_error_codes_without_gpu():
     out = ctypes.c_void_p()
     assert esp.lib.espace_proj_from_device(512, 512, 256, None, None, None, ctypes.byref(out)) == 1
     assert out.value is None
+    # tensor-parallel layers: null pointers, then shapes, are refused before any CUDA call
+    P = np.zeros(4, dtype=np.float64)
+    Pp = P.ctypes.data_as(ctypes.POINTER(ctypes.c_double))
+    fake_w = ctypes.c_void_p(16)
+    assert esp.lib.espace_proj_tp_from_host(esp.TP_ROW, 4, 1024, 512, 64, None, fake_w, None, ctypes.byref(out)) == 1
+    assert esp.lib.espace_proj_tp_from_host(3, 4, 1024, 512, 64, Pp, fake_w, None, ctypes.byref(out)) == 1   # kind
+    assert esp.lib.espace_proj_tp_from_host(esp.TP_ROW, 9, 1152, 512, 64, Pp, fake_w, None, ctypes.byref(out)) == 2
+    assert esp.lib.espace_proj_tp_from_host(esp.TP_ROW, 3, 1008, 512, 64, Pp, fake_w, None, ctypes.byref(out)) == 2
+    assert esp.lib.espace_proj_tp_from_host(esp.TP_ROW, 4, 1024, 512, 320, Pp, fake_w, None, ctypes.byref(out)) == 2
+    assert esp.lib.espace_proj_tp_from_host(esp.TP_COLUMN, 4, 1024, 1000, 64, Pp, fake_w, None, ctypes.byref(out)) == 2
+    assert esp.lib.espace_proj_tp_from_host(esp.TP_COLUMN, 4, 1024, 1024, 96, Pp, fake_w, None, ctypes.byref(out)) == 2
+    assert out.value is None
 
 
 @pytest.mark.parametrize("K", [1, 2, 9, 64, 200])

@@ -278,6 +278,107 @@ def test_single_token_forward_repeated_and_interleaved(esp):
         esp.espace_proj_destroy(p)
 
 
+# ------------------------------------------------------------------ tensor-parallel ranks (Sec. B.2)
+
+TP_CASES = [
+    # (kind, tp, N, K, M, L)
+    ("row", 4, 300, 1024, 776, 128),      # K / tp = 256, ragged M
+    ("row", 3, 129, 576, 392, 64),        # three ranks (K / tp = 192), ragged N
+    ("row", 8, 1000, 2048, 1000, 128),    # eight ranks, several row blocks
+    ("row", 4, 1, 1024, 512, 64),         # one token
+    ("column", 4, 300, 512, 1056, 128),   # M / tp = 264: rank blocks straddle 256-wide tiles
+    ("column", 2, 257, 520, 784, 256),    # K not a multiple of 64, M / tp = 392
+    ("column", 8, 64, 1024, 2048, 64),    # few tokens, eight ranks
+]
+
+
+@pytest.mark.parametrize("kind,tp,N,K,M,L", TP_CASES)
+def test_tp_forward_matches_oracle(esp, kind, tp, N, K, M, L):
+    """Each rank with its own projection: the folded layer (a dense product and a
+    block-diagonal one) against the oracle's per-rank definition."""
+    seed = 3000 + tp + N + K
+    _, X, W = make_layer(K, M, N, seed=seed)
+    r = np.random.default_rng(seed)
+    Kr = K // tp if kind == "row" else K
+    P = np.stack([synth.haar_orthonormal(r, Kr, L) for _ in range(tp)])
+    code = esp.TP_ROW if kind == "row" else esp.TP_COLUMN
+    p = esp.espace_proj_tp_from_host(code, P, dev(W))
+    try:
+        assert esp.espace_proj_tp_info(p) == (code, tp)
+        assert esp.espace_linear_forward_launches(p, N) == 2
+        Y = torch.full((N, M), float("nan"), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Y)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        Pb = oracle.bf16_round(P)
+        bits = esp.espace_proj_read_P(p)
+        assert np.array_equal(synth.bf16_to_f64(torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16)), Pb)
+        Y_o = oracle.forward_tp(f64(X), Pb, f64(W), kind)
+        assert_y_close(Y, Y_o)
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+def test_tp_identity_projections_reproduce_the_dense_layer(esp):
+    """Row-parallel ranks with identity projections (L = K / tp): the folded layer is Eq. 1."""
+    N, K, M, tp = 200, 512, 520, 4
+    _, X, W = make_layer(K, M, N, seed=41)
+    P = np.stack([np.eye(K // tp)] * tp)
+    p = esp.espace_proj_tp_from_host(esp.TP_ROW, P, dev(W))
+    try:
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Y)
+        Yd = torch.empty_like(Y)
+        esp.espace_dense_forward(dev(X), dev(W), Yd)
+        torch.cuda.synchronize()
+        assert_y_close(Y, oracle.dense(f64(X), f64(W)))
+        assert_y_close(Y, f64(Yd))
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+def test_build_projection_tp(esp):
+    """Thm. 1 per rank from one calibration: row-parallel ranks solve C's diagonal blocks
+    (eigenvalues and subspaces against the oracle, then the forward with the library's
+    projections); column-parallel ranks all see C, so the handle is the plain layer."""
+    K, M, L, tp, n, N = 1024, 776, 128, 4, 8192, 300
+    Kr = K // tp
+    model = synth.ActivationModel(K, seed=51, outliers=10, lognormal_sigma=0.5)
+    Xc = model.sample(n, stream="calib_tokens")
+    X = model.sample(N)
+    W = synth.weights(M, K, seed=51)
+    h = esp.espace_calib_create(K)
+    p = q = None
+    try:
+        esp.espace_calib_accumulate(h, dev(Xc))
+        p = esp.espace_build_projection_tp(h, dev(W), L, esp.TP_ROW, tp)
+        assert esp.espace_proj_tp_info(p) == (esp.TP_ROW, tp)
+        w = esp.espace_proj_eigenvalues(p).reshape(tp, Kr)
+        S_o = oracle.autocorr_sum(f64(Xc))
+        P_o, _, w_o = oracle.build_projection_tp(S_o, n, L, "row", tp)
+        Pb = synth.bf16_to_f64(torch.from_numpy(esp.espace_proj_read_P(p).view(np.int16)).view(torch.bfloat16))
+        for r in range(tp):
+            assert np.all(np.diff(w[r]) <= 0)
+            assert np.allclose(w[r], w_o[r], rtol=0, atol=1e-5 * w_o[r][0])
+            gap = w_o[r][L - 1] - w_o[r][L]
+            dC = 1e-5 * np.linalg.norm(S_o / n)
+            proj = np.linalg.norm(Pb[r] @ Pb[r].T - P_o[r] @ P_o[r].T, 2)
+            assert proj <= dC / gap + 2e-2, (r, proj, dC / gap)
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Y)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        assert_y_close(Y, oracle.forward_tp(f64(X), Pb, f64(W), "row"))
+        q = esp.espace_build_projection_tp(h, dev(W), L, esp.TP_COLUMN, tp)
+        assert esp.espace_proj_tp_info(q) == (0, 1)
+        assert esp.espace_proj_shape(q) == (K, M, L)
+    finally:
+        for handle in (p, q):
+            if handle:
+                esp.espace_proj_destroy(handle)
+        esp.espace_calib_destroy(h)
+
+
 @pytest.mark.slow
 def test_llama2_qkv_prefill_full_size_sampled(esp):
     """K=4096, M=12288, L=2048, N=4096 (the benchmark launch): every output of 66 sampled

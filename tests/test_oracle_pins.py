@@ -349,3 +349,91 @@ def test_go_eigenvalues_ordered_by_magnitude():
     assert np.all(np.diff(np.abs(w)) <= 1e-15)
     assert np.allclose(P.T @ P, np.eye(6), atol=1e-12)
     assert np.allclose(P @ np.diag(w) @ P.T, C, atol=1e-12 * np.abs(w).max())
+
+
+# ---------------------------------------------------------------- tensor-parallel ranks (Sec. B.2)
+
+def test_tp_row_brute_force():
+    """Row-parallel ranks, straight from the definition with pure-Python loops: rank r owns
+    the inputs r Kr .. (r+1) Kr - 1, projects them with its own P_r, folds its columns of W
+    with P_r, and the ranks' outputs add up."""
+    r = rng(21)
+    N, K, M, L, tp = 3, 6, 4, 2, 3
+    Kr = K // tp
+    X, W = r.standard_normal((N, K)), r.standard_normal((M, K))
+    P = r.standard_normal((tp, Kr, L))
+    Y = oracle.forward_tp(X, P, W, "row", round_bf16=False)
+    for t in range(N):
+        for m in range(M):
+            ref = 0.0
+            for q in range(tp):
+                for l in range(L):
+                    z = sum(X[t][q * Kr + k] * P[q][k][l] for k in range(Kr))
+                    wf = sum(P[q][k][l] * W[m][q * Kr + k] for k in range(Kr))
+                    ref += z * wf
+            assert abs(Y[t, m] - ref) < 1e-12
+
+
+def test_tp_column_brute_force():
+    """Column-parallel ranks: rank r owns the output rows r Mr .. (r+1) Mr - 1 and projects
+    all K inputs with its own P_r."""
+    r = rng(22)
+    N, K, M, L, tp = 3, 5, 6, 2, 3
+    Mr = M // tp
+    X, W = r.standard_normal((N, K)), r.standard_normal((M, K))
+    P = r.standard_normal((tp, K, L))
+    Y = oracle.forward_tp(X, P, W, "column", round_bf16=False)
+    for t in range(N):
+        for m in range(M):
+            q = m // Mr
+            ref = 0.0
+            for l in range(L):
+                z = sum(X[t][k] * P[q][k][l] for k in range(K))
+                wf = sum(P[q][k][l] * W[m][k] for k in range(K))
+                ref += z * wf
+            assert abs(Y[t, m] - ref) < 1e-12
+
+
+@pytest.mark.parametrize("kind", ["row", "column"])
+def test_tp_identity_projections_reproduce_the_dense_layer(kind):
+    """Full-rank identity projections (L = Kr): every rank passes its inputs through, so the
+    folded layer equals Eq. 1 exactly, bf16 roundings included (they act on bf16 values)."""
+    r = rng(23)
+    N, K, M, tp = 7, 32, 24, 4
+    X = oracle.bf16_round(r.standard_normal((N, K)))
+    W = oracle.bf16_round(r.standard_normal((M, K)) / np.sqrt(K))
+    Kr = K // tp if kind == "row" else K
+    P = np.stack([np.eye(Kr)] * tp)
+    assert np.array_equal(oracle.forward_tp(X, P, W, kind), oracle.dense(X, W))
+
+
+def test_tp_column_with_one_shared_projection_is_the_plain_layer():
+    r = rng(24)
+    N, K, M, L, tp = 5, 16, 12, 6, 4
+    X, W = r.standard_normal((N, K)), r.standard_normal((M, K))
+    P = synth.haar_orthonormal(r, K, L)
+    Y = oracle.forward_tp(X, np.stack([P] * tp), W, "column", round_bf16=False)
+    assert np.allclose(Y, oracle.forward(X, P, W, round_bf16=False)[0], rtol=1e-13, atol=1e-13)
+
+
+def test_tp_row_projections_are_optimal_per_rank():
+    """Thm. 1 applied to each rank's own inputs: rank r's projection MSE on its input slice
+    equals the sum of the discarded eigenvalues of C's r-th diagonal block, which no other
+    L-dimensional projection of that slice beats; the column kind solves the whole C."""
+    r = rng(25)
+    n, K, L, tp = 400, 12, 2, 3
+    Kr = K // tp
+    X = r.standard_normal((n, K)) @ np.diag(np.linspace(2.0, 0.2, K)) @ synth.haar_orthonormal(r, K, K).T
+    S = oracle.autocorr_sum(X)
+    P, _, w = oracle.build_projection_tp(S, n, L, "row", tp)
+    for q in range(tp):
+        Xq = X[:, q * Kr:(q + 1) * Kr]
+        mse = oracle.projection_mse(Xq, P[q])
+        assert abs(mse - np.sum(w[q][L:])) < 1e-10 * np.sum(w[q])
+        for trial in range(20):
+            Q = synth.haar_orthonormal(r, Kr, L)
+            assert oracle.projection_mse(Xq, Q) >= mse - 1e-12
+        assert np.allclose(np.sort(w[q])[::-1], np.linalg.eigvalsh(S[q * Kr:(q + 1) * Kr, q * Kr:(q + 1) * Kr] / n)[::-1])
+    Pc, _, wc = oracle.build_projection_tp(S, n, L, "column", tp)
+    P1, _, w1, _ = oracle.build_projection(S, n, L)
+    assert all(np.array_equal(Pc[q], P1) for q in range(tp)) and np.allclose(wc[0], w1)
