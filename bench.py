@@ -427,6 +427,51 @@ def device_projection(esp, K, L, W, seed):
     return p
 
 
+def tp_projection(esp, kind, tp, K, L, W, seed):
+    """A tensor-parallel handle for timing only: tp seeded random projections folded with W."""
+    Kr = K // tp if kind == "row" else K
+    P = np.random.default_rng(seed).standard_normal((tp, Kr, L)) * Kr ** -0.5
+    return esp.espace_proj_tp_from_host(esp.TP_ROW if kind == "row" else esp.TP_COLUMN, P, W)
+
+
+def table2_rows(esp, peak_tc):
+    """Table 2's per-rank configurations folded onto one GPU, each GEMM of a transformer
+    block timed alone at batch 1 and the model's sequence length (Sec. B.4), dense against
+    ESPACE. Column-parallel ranks calibrated by Thm. 1 share one projection (they see the
+    same inputs), so those layers are the plain projected layer with the rank's L;
+    row-parallel ranks each have their own, which makes the first product block-diagonal."""
+    out = {}
+    seed = synth.BASE_SEED + 700
+    for model, cfg in synth.TABLE2.items():
+        tp, N = cfg["tp"], cfg["seq"]
+        layers = {}
+        for name, kind, K, M, L in cfg["layers"]:
+            W = synth.weights_device(M, K, seed=seed)
+            X = synth.ActivationModel(K, seed=seed).sample_device(N)
+            Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+            per_rank = kind == "row" and tp > 1
+            p = tp_projection(esp, kind, tp, K, L, W, seed) if per_rank else device_projection(esp, K, L, W, seed)
+            try:
+                e_ms = events_ms(lambda i: esp.espace_linear_forward(p, X, Y))
+                d_ms = events_ms(lambda i: esp.espace_dense_forward(X, W, Y))
+                esp.espace_check()
+            finally:
+                esp.espace_proj_destroy(p)
+            width = tp * L if per_rank else L
+            flops = 2.0 * N * (K * width // (tp if per_rank else 1) + width * M)
+            layers[name] = {"kind": kind, "K": K, "M": M, "L_per_rank": L, "tp": tp, "N": N,
+                            "form": "per-rank block-diagonal" if per_rank else "plain", "espace_ms": e_ms,
+                            "dense_ms": d_ms, "espace_tflops": flops / e_ms / 1e9,
+                            "dense_tflops": 2.0 * N * K * M / d_ms / 1e9}
+            del W, X, Y
+        e_tot = sum(v["espace_ms"] for v in layers.values())
+        d_tot = sum(v["dense_ms"] for v in layers.values())
+        out[model] = {"layers": layers, "espace_ms": e_tot, "dense_ms": d_tot,
+                      "gemm_latency_reduction": 1.0 - e_tot / d_tot,
+                      "paper_reduction_a100": cfg["paper_reduction"]}
+    return out
+
+
 def layer_row(esp, K, M, L, N, seed, peak_tc):
     """One layer at N tokens: the projected forward and the dense one (inputs larger than L2
     are read by every call, so no rotation is needed)."""
@@ -534,6 +579,7 @@ def config_rows(esp, peak_tc, peak_hbm):
                       "dense_ms": sum(v["dense_ms"] for v in layer.values())}
     layer["total"]["speedup"] = layer["total"]["dense_ms"] / layer["total"]["espace_ms"]
     rows["llama2_layer_prefill_batch1_seq4096"] = layer
+    rows["table2_tp_folded_gemm_latency"] = table2_rows(esp, peak_tc)
     return rows
 
 

@@ -900,6 +900,20 @@ static int tp_forward(espace_proj_s* p, const void* X, int n, void* Y, cudaStrea
 // CTA-pair launch).
 static bool swap_forward_applies(int n, int path) { return n <= SWAP_MAX_TOKENS && path != ESPACE_PATH_TENSOR_SPLIT; }
 
+// Above SWAP_MAX_TOKENS, a rank-L product with fewer 256 x 256 tiles than a quarter of the
+// SMs (small L and N, e.g. L = 512 at 2048 tokens: 16 tiles) leaves most CTA pairs of the
+// fused launch idle while it runs. When it also holds most of the work (K >= 2 M, e.g. an
+// FC2 layer) it takes the swapped product with its reduction split over the SMs instead,
+// then the folded-weight product on CTA pairs (measured: GPT3-1.3B FC2 at 2048 tokens 56 ->
+// 42 us); otherwise the fused launch, whose folded-weight tiles fill the idle pairs, stays
+// faster (GPT3-1.3B QKV 41 against 47 us, GPT3-8B QKV 73 against 86 us).
+static bool split_phase1_applies(int n, int K, int Lp, int M, int num_sms, int path)
+{
+    const int64_t tiles = ((static_cast<int64_t>(n) + 255) / 256) * ((Lp + 255) / 256);
+    return n > SWAP_MAX_TOKENS && path != ESPACE_PATH_SMALL_N && tiles < num_sms / 4 &&
+           static_cast<int64_t>(K) >= 2 * static_cast<int64_t>(M);
+}
+
 int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev, void* stream,
                                int path)
 {
@@ -941,6 +955,12 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
         CUDA_TRY(launch_gemm_swap(p->PT, K, X_dev, K, Lp, n, K, p->Z, Lp, p->part, st), "forward: phase 1");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
         CUDA_TRY(launch_gemm_swap(p->WfT, Lp, p->Z, Lp, M, n, Lp, Y_dev, M, p->part, st), "forward: phase 2");
+    } else if (split_phase1_applies(n, K, Lp, M, dev->num_sms, path)) {
+        rc = ensure_swap(p, n, dev->num_sms, st);
+        if (rc != ESPACE_OK) return rc;
+        CUDA_TRY(launch_gemm_swap(p->PT, K, X_dev, K, Lp, n, K, p->Z, Lp, p->part, st), "forward: phase 1");
+        if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
+        CUDA_TRY(launch_gemm_tn(p->Z, Lp, p->WfT, Lp, n, M, Lp, Y_dev, M, st), "forward: phase 2");
     } else if (path != ESPACE_PATH_TENSOR_SPLIT && fused_forward_applies(n, Lp, M)) {
         // one persistent launch holds both products; the phase event marks its start
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
@@ -976,6 +996,8 @@ int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path)
         const int b = gemm_swap_plan(M, n, Lp, dev->num_sms, true).ksplit > 1 ? 2 : 1;
         return a + b;
     }
+    if (split_phase1_applies(n, K, Lp, M, dev->num_sms, path))
+        return (gemm_swap_plan(Lp, n, K, dev->num_sms, true).ksplit > 1 ? 2 : 1) + 1;
     if (path != ESPACE_PATH_TENSOR_SPLIT && fused_forward_applies(n, Lp, M)) return 1;
     return 2;
 }

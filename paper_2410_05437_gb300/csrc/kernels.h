@@ -31,11 +31,13 @@ cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ld
 cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,
                                  int K, int Lp, int M, int* ready, int* done, cudaStream_t stream);
 
-// Swapped product for few tokens (ntok <= 256): out[n][r] (bf16, leading dimension ldo) =
-// sum_k W[r][k] X[n][k], the weights as the 128-row tcgen05 operand, the tile stored
-// transposed. The reduction splits over CTAs (ksplit > 1) only when a workspace `part` of
-// the plan's part_elems fp32 values (made with allow_split) is given; a second launch then
-// adds the partials in split order.
+// Swapped product: out[n][r] (bf16, leading dimension ldo) = sum_k W[r][k] X[n][k], the
+// weights as the 128-row tcgen05 operand, the tile stored transposed, token tiles of 128
+// (ntok <= 128) or 256. The reduction splits over CTAs (ksplit > 1) when the tiles would
+// leave more than half of the SMs idle and a workspace `part` of the plan's part_elems
+// fp32 values (made with allow_split) is given; a second launch then adds the partials in
+// split order. Used for few tokens (ntok <= SWAP_MAX_TOKENS), and for the rank-L product of
+// a layer whose Z has too few 256 x 256 tiles to occupy the CTA pairs.
 struct SwapPlan {
     int bn = 128, tiles = 0, kblocks = 0, ksplit = 1, kb_per_split = 0;
     int64_t ld_part = 0, part_elems = 0;

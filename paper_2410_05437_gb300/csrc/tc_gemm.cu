@@ -1064,7 +1064,6 @@ cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t 
                              void* out, int64_t ldo, float* part, cudaStream_t stream)
 {
     if (rows <= 0 || ntok <= 0) return cudaSuccess;
-    if (ntok > 256) return cudaErrorInvalidValue;
     DeviceInfo* dev = nullptr;
     if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
     // without a workspace the reduction is not split

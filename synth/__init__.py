@@ -224,6 +224,33 @@ DECODE_LAYERS = {
 }
 DECODE_TOKENS = (1, 8, 32, 128, 512)
 
+# Per-layer ESPACE configurations of Table 2 (Sec. B.2): per model the tensor-parallel rank
+# count, the sequence length of the GEMM latency measurement (Sec. B.4: batch 1, 2048
+# tokens for GPT3, 4096 for Llama2 and Nemotron4), and per layer (name, kind, K, M, L)
+# with K, M the whole layer's input and output widths and L the per-rank rank; QKV and
+# FC1 are column-parallel, the attention projection and FC2 row-parallel. Also Table 1's
+# total GEMM latency reduction of the most compressed variant, on A100.
+TABLE2 = {
+    "gpt3_1.3b": dict(tp=1, seq=2048, paper_reduction=0.34, layers=[
+        ("qkv", "column", 2048, 6144, 512), ("proj", "row", 2048, 2048, 512),
+        ("fc1", "column", 2048, 8192, 512), ("fc2", "row", 8192, 2048, 512)]),
+    "gpt3_8b": dict(tp=4, seq=2048, paper_reduction=0.44, layers=[
+        ("qkv", "column", 4096, 12288, 1024), ("proj", "row", 4096, 4096, 256),
+        ("fc1", "column", 4096, 16384, 1024), ("fc2", "row", 16384, 4096, 1024)]),
+    "gpt3_22b": dict(tp=8, seq=2048, paper_reduction=0.49, layers=[
+        ("qkv", "column", 6144, 18432, 2048), ("proj", "row", 6144, 6144, 256),
+        ("fc1", "column", 6144, 24576, 2048), ("fc2", "row", 24576, 6144, 1024)]),
+    "llama2_7b": dict(tp=4, seq=4096, paper_reduction=0.46, layers=[
+        ("qkv", "column", 4096, 12288, 1024), ("proj", "row", 4096, 4096, 256),
+        ("fc1", "column", 4096, 22016, 1024), ("fc2", "row", 11008, 4096, 512)]),
+    "llama2_13b": dict(tp=8, seq=4096, paper_reduction=0.36, layers=[
+        ("qkv", "column", 5120, 15360, 2048), ("proj", "row", 5120, 5120, 256),
+        ("fc1", "column", 5120, 27648, 2048), ("fc2", "row", 13824, 5120, 1024)]),
+    "nemotron4_15b": dict(tp=8, seq=4096, paper_reduction=0.46, layers=[
+        ("qkv", "column", 6144, 8192, 2048), ("proj", "row", 6144, 6144, 256),
+        ("fc1", "column", 6144, 24576, 2048), ("fc2", "row", 24576, 6144, 1024)]),
+}
+
 
 def config_seed(name: str) -> int:
     return BASE_SEED + list(CONFIGS).index(name)

@@ -136,6 +136,9 @@ FORWARD_CASES = [
     (600, 1024, 1000, 512, 1),     # one persistent launch for both products, ragged M
     (600, 1024, 1000, 512, 3),     # the same on two launches
     (1000, 2048, 2312, 1000, 1),   # fused, ragged N / L / M, several row blocks
+    (777, 2048, 1000, 256, 0),     # K >= 2 M and few Z tiles: rank-L product split over the SMs
+    (300, 1040, 264, 64, 1),       # the same just above the swapped token range, ragged K
+    (2304, 1152, 520, 1152, 1),    # 45 Z tiles: one persistent launch for both products
     (300, 1024, 3000, 300, 3),
     # few tokens on tcgen05 with the weights as the 128-row operand; split reductions
     (100, 4096, 776, 2048, 1),     # both products split (16 and 7 weight tiles)
@@ -166,6 +169,16 @@ def test_launch_counts(esp):
         # followed by the launch that adds the partials
         assert esp.espace_linear_forward_launches(p, 100, esp.PATH_TENSOR) == 4
         assert esp.espace_linear_forward_launches(p, 64, esp.PATH_SMALL_N) == -1
+    finally:
+        esp.espace_proj_destroy(p)
+    # K >= 2 M with 12 Z tiles at 600 tokens: the rank-L product splits its reduction (one
+    # launch for the partials, one adding them), then the folded-weight product
+    K, M, L = 2048, 1000, 512
+    p = esp.espace_proj_from_host(synth.random_projection(K, L, seed=3), dev(synth.weights(M, K, seed=3)))
+    try:
+        assert esp.espace_linear_forward_launches(p, 600) == 3
+        assert esp.espace_linear_forward_launches(p, 600, esp.PATH_TENSOR_SPLIT) == 3
+        assert esp.espace_linear_forward_launches(p, 4864) == 1      # 38 Z tiles: fused
     finally:
         esp.espace_proj_destroy(p)
 
