@@ -78,6 +78,20 @@ int espace_calib_accumulate(espace_calib_t h, const void* X_dev, int64_t N, void
 int espace_calib_accumulate_normalized(espace_calib_t h, const void* X_dev, int64_t N,
                                        void* stream);
 
+/* Async. Thm. 2's NL-MSE calibration (Sec. 3.3, App. A.4): for one calibration sequence of
+ * T tokens with activations X_dev ([T][K] bf16) and the loss gradients with respect to them
+ * G_dev ([T][K] bf16), adds C_i = (A B + B A) / T^2, A = X^T X, B = G^T G, to the
+ * accumulator and counts one sequence (the paper's per-sequence approximation; C = S / n is
+ * then the mean over sequences). normalized != 0 takes the L2-normalized variant (every
+ * token row of X and of G divided by its norm first). A and B are formed on the tensor
+ * cores (fp32), each split into bf16 hi + lo halves, and the products accumulated as
+ * A_hi B_hi + A_hi B_lo + A_lo B_hi (and the same for B A) in fp32: about 2^-16 relative.
+ * Cannot be mixed with the other accumulations on one handle (ESPACE_ERR_STATE). The first
+ * call allocates 16 K^2 bytes of scratch on the handle (4 T K bytes more when normalized).
+ * C may be indefinite: espace_build_projection then orders eigenvalues by magnitude. */
+int espace_calib_accumulate_nl(espace_calib_t h, const void* X_dev, const void* G_dev, int64_t T,
+                               int normalized, void* stream);
+
 /* Synchronizes `stream`, then writes C = S / n as a full symmetric K x K fp64 matrix
  * (C_host may be NULL) and the token count (n_out may be NULL). ESPACE_ERR_STATE if n = 0
  * and C_host != NULL. */
@@ -102,7 +116,9 @@ void espace_calib_destroy(espace_calib_t h);
 /* Synchronous. Builds the projected layer from a calibrated accumulator:
  *   1. C = S / n in fp64 on the host;
  *   2. symmetric eigen-decomposition of C in fp64 on the host (Householder
- *      tridiagonalization and implicit QR), eigenvalues sorted decreasing (Sec. 3.1);
+ *      tridiagonalization and implicit QR), eigenvalues sorted decreasing (Sec. 3.1), or
+ *      by decreasing magnitude when C is not positive semidefinite (smallest eigenvalue
+ *      below -1e-6 of the largest magnitude; e.g. an NL-MSE matrix), as the paper does;
  *   3. P = the first L eigenvectors (Thm. 1), each column's largest-magnitude entry made
  *      positive (lowest index on ties), rounded to bf16;
  *   4. W'^T = W P rounded to bf16, i.e. W' = P^T W (Sec. 2.2), on the GPU with fp32
@@ -189,11 +205,12 @@ int espace_proj_tp_from_host(int kind, int tp, int64_t K, int64_t M, int64_t L, 
                              const void* W_dev, void* stream, espace_proj_t* out);
 
 /* Synchronous. As espace_build_projection (Thm. 1 per rank) for a tensor-parallel layer:
- * rank r's autocorrelation is that of its own inputs, i.e. C = S / n for COLUMN (every rank
- * sees all K inputs, so the ranks' projections coincide and the returned handle is the
- * plain layer with the rank's L; the paper's per-rank L, Table 2) and the r-th diagonal
- * K/tp x K/tp block of C for ROW (tp eigen-solves of size K / tp; the handle's
- * eigenvalues are the tp ranks' K / tp values, each block decreasing). */
+ * rank r's autocorrelation is that of its own inputs. ROW: the r-th diagonal K/tp x K/tp
+ * block of C = S / n (tp eigen-solves of size K / tp; the handle's eigenvalues are the tp
+ * ranks' K / tp values, each block decreasing). COLUMN: every rank sees all K inputs, so
+ * the ranks' projections coincide and the call is espace_build_projection with the rank's
+ * L (Table 2's per-rank L), returning a plain handle; only tp's range is checked. Needs a
+ * plain or normalized activation accumulation (ESPACE_ERR_STATE after NL-MSE). */
 int espace_build_projection_tp(espace_calib_t h, const void* W_dev, int64_t M, int64_t L, int kind, int tp,
                                void* stream, espace_proj_t* out);
 

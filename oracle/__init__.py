@@ -20,7 +20,10 @@ arrays and chains the steps in the order the paper states them:
 * ``go_mse_matrix`` / ``build_projection_go``  Thm. 2: C = C_X C_W + C_W C_X, P its L
   principal eigenvectors (ordered by |eigenvalue|, as the paper does when C is indefinite);
 * ``forward_tp`` / ``build_projection_tp``  ESPACE applied per tensor-parallel rank
-  (Sec. B.2, Table 2), the ranks folded onto one device (Sec. B.4).
+  (Sec. B.2, Table 2), the ranks folded onto one device (Sec. B.4);
+* ``nl_mse_term`` / ``order_eigenpairs``  Thm. 2's NL-MSE matrix for one calibration
+  sequence (App. A.4's per-sequence form) and the eigenvalue order the paper uses when a
+  calibrated C is not positive definite.
 
 Layout: tokens are rows (``X`` is ``[N, K]``), ``W`` is ``[M, K]`` as in ``nn.Linear``,
 ``P`` is ``[K, L]``, ``W'`` is ``[L, M]``, ``Z`` is ``[N, L]`` and ``Y`` is ``[N, M]``.
@@ -285,3 +288,34 @@ def build_projection_tp(S, n: int, L: int, kind: str, tp: int):
         Sr = S if kind == "column" else S[r * Kr:(r + 1) * Kr, r * Kr:(r + 1) * Kr]
         P[r], _, w[r], _ = build_projection(Sr, n, L)
     return P, bf16_round(P), w
+
+
+def nl_mse_term(X, G, normalized: bool = False) -> np.ndarray:
+    """Thm. 2, NL-MSE, in App. A.4's per-sequence form: for one calibration sequence of T
+    tokens (rows of ``X``) and the loss gradients with respect to them (rows of ``G``),
+    ``C_i = (X^T X G^T G + G^T G X^T X) / T^2``; C is the mean of C_i over sequences. With
+    ``normalized`` the L2-normalized variant of Sec. 3.3: every row of X and of G is
+    divided by its norm first (a zero row stays zero)."""
+    X, G = _f64(X), _f64(G)
+    T = X.shape[0]
+    assert G.shape == X.shape
+    if normalized:
+        nx = np.linalg.norm(X, axis=1, keepdims=True)
+        ng = np.linalg.norm(G, axis=1, keepdims=True)
+        X = np.where(nx > 0, X / np.where(nx > 0, nx, 1.0), 0.0)
+        G = np.where(ng > 0, G / np.where(ng > 0, ng, 1.0), 0.0)
+    A = autocorr_sum(X)
+    B = autocorr_sum(G)
+    return (A @ B + B @ A) / float(T) ** 2
+
+
+def order_eigenpairs(w, V, tol: float = 1e-6):
+    """Eigenvalues decreasing (Sec. 3.1); when C is not positive semidefinite -- its smallest
+    eigenvalue below ``-tol`` times the largest magnitude, a margin for rounding -- by
+    decreasing magnitude instead, as the paper does (ties keep the decreasing order).
+    ``w`` decreasing as ``eigh`` returns it; returns the reordered ``(w, V)``."""
+    w, V = np.asarray(w), np.asarray(V)
+    if w[-1] < -tol * np.abs(w).max():
+        order = np.argsort(-np.abs(w), kind="stable")
+        return w[order], V[:, order]
+    return w, V

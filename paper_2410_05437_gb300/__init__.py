@@ -34,6 +34,7 @@ __all__ = [
     "espace_host_eigh",
     "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "PATH_TENSOR_SPLIT", "EXPORTED_SYMBOLS",
     "TP_COLUMN", "TP_ROW", "espace_proj_tp_from_host", "espace_build_projection_tp", "espace_proj_tp_info",
+    "espace_calib_accumulate_nl",
     "espace_linear_forward_launches",
 ]
 
@@ -71,6 +72,7 @@ _SIGNATURES = {
     "espace_calib_create": (ctypes.c_int, [_i64, ctypes.POINTER(_vp)]),
     "espace_calib_accumulate": (ctypes.c_int, [_vp, _vp, _i64, _vp]),
     "espace_calib_accumulate_normalized": (ctypes.c_int, [_vp, _vp, _i64, _vp]),
+    "espace_calib_accumulate_nl": (ctypes.c_int, [_vp, _vp, _vp, _i64, ctypes.c_int, _vp]),
     "espace_calib_read": (ctypes.c_int, [_vp, _pd, _pi64, _vp]),
     "espace_calib_export": (ctypes.c_int, [_vp, _pf, _pi64, _vp]),
     "espace_calib_import": (ctypes.c_int, [_vp, _pf, _i64, _vp]),
@@ -192,6 +194,14 @@ def espace_calib_accumulate(h: int, X, N: int | None = None, stream=None) -> Non
 def espace_calib_accumulate_normalized(h: int, X, N: int | None = None, stream=None) -> None:
     N = X.shape[0] if N is None else N
     _check(lib.espace_calib_accumulate_normalized(h, _dev_ptr(X), int(N), _stream(stream)))
+
+
+def espace_calib_accumulate_nl(h: int, X, G, normalized: bool = False, stream=None) -> None:
+    """One NL-MSE calibration sequence: X, G device bf16 [T][K] (activations and the loss
+    gradients with respect to them)."""
+    assert tuple(X.shape) == tuple(G.shape)
+    _check(lib.espace_calib_accumulate_nl(h, _dev_ptr(X), _dev_ptr(G), int(X.shape[0]), int(bool(normalized)),
+                                          _stream(stream)))
 
 
 def espace_calib_read(h: int, K: int, stream=None):

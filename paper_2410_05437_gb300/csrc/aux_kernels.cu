@@ -75,6 +75,29 @@ cudaError_t launch_sym_full_f64(const float* Su, int64_t K, double scale, double
     return cudaGetLastError();
 }
 
+__global__ void sym_split_bf16_kernel(const float* __restrict__ Su, int64_t K, float scale,
+                                      __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo)
+{
+    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < K * K;
+         e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t i = e / K, j = e - i * K;
+        const float v = scale * (i <= j ? Su[i * K + j] : Su[j * K + i]);
+        const __nv_bfloat16 h = __float2bfloat16_rn(v);
+        hi[e] = h;
+        // v - h is exact in fp32 (h is v rounded to 8 significant bits)
+        lo[e] = __float2bfloat16_rn(v - __bfloat162float(h));
+    }
+}
+
+cudaError_t launch_sym_split_bf16(const float* Su, int64_t K, float scale, void* hi, void* lo, cudaStream_t stream)
+{
+    if (K <= 0) return cudaSuccess;
+    const int64_t blocks = std::min<int64_t>((K * K + 255) / 256, 65536);
+    sym_split_bf16_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+        Su, K, scale, static_cast<__nv_bfloat16*>(hi), static_cast<__nv_bfloat16*>(lo));
+    return cudaGetLastError();
+}
+
 // T = A B for K x K row-major fp64 matrices: 64 x 64 output tiles, 256 threads with 4 x 4
 // outputs each, 16-deep slices of A and B staged in shared memory; each output summed in
 // k order.

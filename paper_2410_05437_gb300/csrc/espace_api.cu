@@ -168,9 +168,14 @@ struct espace_calib_s {
     int device = 0;
     float* S = nullptr;            // [K][K] fp32, upper triangle valid
     int64_t n = 0;
-    int mode = 0;                  // 0 unset, 1 plain, 2 normalized (Cor. 1)
+    int mode = 0;                  // 0 unset, 1 plain, 2 normalized (Cor. 1), 3 NL-MSE (Thm. 2),
+                                   // 4 NL-MSE with L2-normalized tokens and gradients
     void* xn = nullptr;            // scratch for normalized tokens
     int64_t xn_tokens = 0;
+    void* gn = nullptr;            // scratch for normalized gradients (NL-MSE)
+    int64_t gn_tokens = 0;
+    float* nl_f32 = nullptr;       // NL-MSE scratch: two K x K fp32 autocorrelations
+    void* nl_bf = nullptr;         //   and four K x K bf16 halves (hi / lo of each)
 };
 
 struct espace_proj_s {
@@ -307,6 +312,79 @@ int espace_calib_accumulate_normalized(espace_calib_t h, const void* X_dev, int6
     return calib_accumulate_impl(h, X_dev, N, stream, 2);
 }
 
+// Grows a bf16 token scratch of the calibration handle to `tokens` rows (synchronously).
+static int grow_token_scratch(espace_calib_t h, void** buf, int64_t* cap, int64_t tokens, cudaStream_t st)
+{
+    if (*cap >= tokens) return ESPACE_OK;
+    CUDA_TRY(cudaStreamSynchronize(st), "calibration scratch: sync");
+    if (*buf) cudaFree(*buf);
+    *buf = nullptr;
+    *cap = 0;
+    cudaError_t e = cudaMalloc(buf, sizeof(uint16_t) * tokens * h->K);
+    if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "calibration scratch: %s", cudaGetErrorString(e));
+    *cap = tokens;
+    return ESPACE_OK;
+}
+
+int espace_calib_accumulate_nl(espace_calib_t h, const void* X_dev, const void* G_dev, int64_t T, int normalized,
+                               void* stream)
+{
+    if (h == nullptr) return fail(ESPACE_ERR_ARG, "espace_calib_accumulate_nl: null handle");
+    if (X_dev == nullptr || G_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_calib_accumulate_nl: null pointer");
+    if (T < 1 || T > (int64_t(1) << 31) - 64)
+        return fail(ESPACE_ERR_SHAPE, "espace_calib_accumulate_nl: T=%lld tokens", (long long)T);
+    if (!aligned16(X_dev) || !aligned16(G_dev))
+        return fail(ESPACE_ERR_ALIGN, "espace_calib_accumulate_nl: X / G not 16-byte aligned");
+    const int mode = normalized ? 4 : 3;
+    if (h->mode != 0 && h->mode != mode)
+        return fail(ESPACE_ERR_STATE, "espace_calib_accumulate_nl: mixed with another accumulation on one handle");
+    DeviceGuard g(h->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t K = h->K, kk = K * K;
+    if (normalized) {
+        // the L2-normalized variant: x / |x| and g / |g| for every token (Sec. 3.3)
+        int rc = grow_token_scratch(h, &h->xn, &h->xn_tokens, T, st);
+        if (rc == ESPACE_OK) rc = grow_token_scratch(h, &h->gn, &h->gn_tokens, T, st);
+        if (rc != ESPACE_OK) return rc;
+        CUDA_TRY(launch_normalize_rows(X_dev, T, static_cast<int>(K), h->xn, st), "accumulate_nl: normalize X");
+        CUDA_TRY(launch_normalize_rows(G_dev, T, static_cast<int>(K), h->gn, st), "accumulate_nl: normalize G");
+        X_dev = h->xn;
+        G_dev = h->gn;
+    }
+    if (h->nl_f32 == nullptr) {
+        cudaError_t e = cudaMalloc(&h->nl_f32, sizeof(float) * 2 * kk);
+        if (e == cudaSuccess) e = cudaMalloc(&h->nl_bf, sizeof(uint16_t) * 4 * kk);
+        if (e != cudaSuccess) {
+            if (h->nl_f32) cudaFree(h->nl_f32);
+            h->nl_f32 = nullptr;
+            h->nl_bf = nullptr;
+            return fail(ESPACE_ERR_NOMEM, "espace_calib_accumulate_nl: scratch: %s", cudaGetErrorString(e));
+        }
+    }
+    float* a32 = h->nl_f32;
+    float* b32 = h->nl_f32 + kk;
+    uint16_t* a_hi = static_cast<uint16_t*>(h->nl_bf);
+    uint16_t* a_lo = a_hi + kk;
+    uint16_t* b_hi = a_lo + kk;
+    uint16_t* b_lo = b_hi + kk;
+    const int k = static_cast<int>(K);
+    // A = X^T X / T and B = G^T G / T (upper triangles on the tensor cores, then the full
+    // symmetric matrices split into bf16 hi + lo)
+    CUDA_TRY(launch_zero_f32(h->nl_f32, 2 * kk, st), "accumulate_nl: clear");
+    CUDA_TRY(launch_syrk_upper(X_dev, T, k, a32, st), "accumulate_nl: X^T X");
+    CUDA_TRY(launch_syrk_upper(G_dev, T, k, b32, st), "accumulate_nl: G^T G");
+    CUDA_TRY(launch_sym_split_bf16(a32, K, 1.0f / static_cast<float>(T), a_hi, a_lo, st), "accumulate_nl: split A");
+    CUDA_TRY(launch_sym_split_bf16(b32, K, 1.0f / static_cast<float>(T), b_hi, b_lo, st), "accumulate_nl: split B");
+    // S += (A B + B A), upper triangle: A B ~ A_hi B_hi + A_hi B_lo + A_lo B_hi and the same
+    // for B A; A and B are symmetric, so S += U^T V with U, V one of them each is S += U V
+    const uint16_t* pairs[6][2] = {{a_hi, b_hi}, {a_hi, b_lo}, {a_lo, b_hi}, {b_hi, a_hi}, {b_hi, a_lo}, {b_lo, a_hi}};
+    for (auto& pr : pairs)
+        CUDA_TRY(launch_syrk_cross_upper(pr[0], pr[1], K, k, h->S, st), "accumulate_nl: product");
+    h->mode = mode;
+    h->n += 1;
+    return ESPACE_OK;
+}
+
 static int read_sum(espace_calib_t h, std::vector<float>& S, void* stream)
 {
     DeviceGuard g(h->device);
@@ -382,6 +460,9 @@ void espace_calib_destroy(espace_calib_t h)
     cudaDeviceSynchronize();
     if (h->S) cudaFree(h->S);
     if (h->xn) cudaFree(h->xn);
+    if (h->nl_f32) cudaFree(h->nl_f32);
+    if (h->nl_bf) cudaFree(h->nl_bf);
+    if (h->gn) cudaFree(h->gn);
     delete h;
 }
 
@@ -471,6 +552,7 @@ int espace_build_projection_go(espace_calib_t h, const void* W_dev, int64_t M, i
     if (rc != ESPACE_OK) return rc;
     if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_build_projection_go: W not 16-byte aligned");
     if (h->n == 0) return fail(ESPACE_ERR_STATE, "espace_build_projection_go: no calibration tokens");
+    if (h->mode > 2) return fail(ESPACE_ERR_STATE, "espace_build_projection_go: needs an activation autocorrelation");
     DeviceGuard g(h->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const size_t kk = static_cast<size_t>(K * K);
@@ -566,9 +648,19 @@ int espace_build_projection(espace_calib_t h, const void* W_dev, int64_t M, int6
     mirror_scaled(S, K, 1.0 / static_cast<double>(h->n), C.data());
     rc = host_eigh(C.data(), K, w.data(), V.data(), 0);
     if (rc != ESPACE_OK) return fail(rc, "espace_build_projection: eigen-solver did not converge");
-    std::vector<double> P(static_cast<size_t>(K * L));
+    // decreasing eigenvalues; when C is not positive semidefinite (e.g. an NL-MSE matrix),
+    // decreasing |eigenvalue| instead, as the paper does (ties keep the signed order)
+    std::vector<int64_t> order(K);
+    for (int64_t i = 0; i < K; ++i) order[i] = i;
+    const double wmax = std::max(std::fabs(w[0]), std::fabs(w[K - 1]));
+    if (w[K - 1] < -1e-6 * wmax)
+        std::stable_sort(order.begin(), order.end(),
+                         [&](int64_t a, int64_t b) { return std::fabs(w[a]) > std::fabs(w[b]); });
+    std::vector<double> P(static_cast<size_t>(K * L)), wo(K);
+    for (int64_t i = 0; i < K; ++i) wo[i] = w[order[i]];
+    w = wo;
     for (int64_t k = 0; k < K; ++k)
-        for (int64_t l = 0; l < L; ++l) P[k * L + l] = V[k * K + l];
+        for (int64_t l = 0; l < L; ++l) P[k * L + l] = V[k * K + order[l]];
     espace_proj_s* p = nullptr;
     rc = proj_create(K, M, L, &p);
     if (rc != ESPACE_OK) return rc;
@@ -675,12 +767,16 @@ int espace_build_projection_tp(espace_calib_t h, const void* W_dev, int64_t M, i
         return fail(ESPACE_ERR_ARG, "espace_build_projection_tp: null pointer");
     *out = nullptr;
     const int64_t K = h->K;
+    if (kind == ESPACE_TP_COLUMN) {
+        if (tp < 1 || tp > 8) return fail(ESPACE_ERR_SHAPE, "tensor parallel: tp=%d must be in [1, 8]", tp);
+        // every column-parallel rank sees all K inputs: one eigen-solve, the plain layer
+        return espace_build_projection(h, W_dev, M, L, stream, out);
+    }
     int rc = check_tp_shape(kind, tp, K, M, L);
     if (rc != ESPACE_OK) return rc;
-    // every column-parallel rank sees all K inputs: one eigen-solve, the plain layer
-    if (kind == ESPACE_TP_COLUMN) return espace_build_projection(h, W_dev, M, L, stream, out);
     if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_build_projection_tp: W not 16-byte aligned");
     if (h->n == 0) return fail(ESPACE_ERR_STATE, "espace_build_projection_tp: no calibration tokens");
+    if (h->mode > 2) return fail(ESPACE_ERR_STATE, "espace_build_projection_tp: needs an activation autocorrelation");
     DeviceGuard g(h->device);
     std::vector<float> S;
     rc = read_sum(h, S, stream);

@@ -62,6 +62,8 @@ cudaError_t launch_gemm_tn_blocks(const void* A, int64_t lda, int a_cols, const 
 
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
+// The same kernel with two operands: S's upper triangle += that of X^T Y (X, Y [N][K] bf16).
+cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream);
 
 // Token counts served by the decode kernels (when asked for), and chosen for them by the
 // automatic paths: above these, the swapped tcgen05 products measured faster.
@@ -92,6 +94,9 @@ cudaError_t launch_wait_timeout(uint64_t limit_ns, cudaStream_t stream);
 
 // C[K][K] (fp64) = scale * (the symmetric matrix whose upper triangle is Su, fp32).
 cudaError_t launch_sym_full_f64(const float* Su, int64_t K, double scale, double* C, cudaStream_t stream);
+// The symmetric matrix whose upper triangle is Su (fp32, K x K), times scale, split into two
+// bf16 matrices: hi = bf16(v), lo = bf16(v - hi), so that hi + lo carries 16 significant bits.
+cudaError_t launch_sym_split_bf16(const float* Su, int64_t K, float scale, void* hi, void* lo, cudaStream_t stream);
 // T = A B for K x K row-major fp64 matrices.
 cudaError_t launch_gemm_f64(const double* A, const double* B, int K, double* T, cudaStream_t stream);
 

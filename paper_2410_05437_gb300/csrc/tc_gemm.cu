@@ -1180,6 +1180,11 @@ void choose_splits(int kblocks, int tiles, int workers, int* ksplit, int* kb_per
 
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream)
 {
+    return launch_syrk_cross_upper(X, X, N, K, S, stream);
+}
+
+cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream)
+{
     if (N <= 0) return cudaSuccess;
     DeviceInfo* dev = nullptr;
     if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
@@ -1191,7 +1196,9 @@ cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStr
         if (tiles == nullptr) return cudaErrorMemoryAllocation;
         CUtensorMap maps[4];
         if (!encode_map(&maps[0], X, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
-        maps[1] = maps[2] = maps[3] = maps[0];
+        if (!encode_map(&maps[1], Y, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
+        maps[2] = maps[0];
+        maps[3] = maps[1];
         PairArgs a{};
         PairProblem& p = a.p[0];
         p.rows = K;
@@ -1211,8 +1218,9 @@ cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStr
     int count = 0;
     const int2* tiles = syrk_tiles(K, BM, 256, &count);
     if (tiles == nullptr) return cudaErrorMemoryAllocation;
-    CUtensorMap mx;
+    CUtensorMap mx, my;
     if (!encode_map(&mx, X, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
+    if (!encode_map(&my, Y, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
     TcGemmArgs a{};
     a.rows = K;
     a.cols = K;
@@ -1229,7 +1237,7 @@ cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStr
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
     const int grid = std::min(a.num_tiles * a.ksplit, dev->num_sms);
-    return launch_kernel<256, 4, true, EPI_ATOMIC_UPPER_F32>(mx, mx, a, grid, stream);
+    return launch_kernel<256, 4, true, EPI_ATOMIC_UPPER_F32>(mx, my, a, grid, stream);
 }
 
 cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,

@@ -291,6 +291,68 @@ def test_single_token_forward_repeated_and_interleaved(esp):
         esp.espace_proj_destroy(p)
 
 
+# ------------------------------------------------------------------ NL-MSE calibration (Thm. 2)
+
+def _unit_rows_bf16(A):
+    A = f64(A)
+    n = np.linalg.norm(A, axis=1, keepdims=True)
+    return oracle.bf16_round(np.where(n > 0, A / np.where(n > 0, n, 1.0), 0.0))
+
+
+@pytest.mark.parametrize("normalized", [False, True])
+def test_calib_nl_mse_matches_oracle(esp, normalized):
+    """Three calibration sequences of activations and synthetic loss gradients: C (the mean
+    of the per-sequence NL-MSE matrices) against the oracle, then the projection (ordered
+    by |eigenvalue| when C is indefinite) and the forward with the library's P."""
+    K, M, L, T, nseq, N = 512, 512, 128, 256, 3, 96
+    xm = synth.ActivationModel(K, seed=61, outliers=5, lognormal_sigma=0.5)
+    gm = synth.ActivationModel(K, seed=62, outliers=0, lognormal_sigma=0.0)
+    Xs = [xm.sample(T, stream="calib_tokens", chunk=i) for i in range(nseq)]
+    Gs = [gm.sample(T, stream="calib_tokens", chunk=i) * 0.01 for i in range(nseq)]
+    Gs = [g.to(torch.bfloat16) for g in Gs]
+    X = xm.sample(N)
+    W = synth.weights(M, K, seed=61)
+    h = esp.espace_calib_create(K)
+    p = None
+    try:
+        for Xi, Gi in zip(Xs, Gs):
+            esp.espace_calib_accumulate_nl(h, dev(Xi), dev(Gi), normalized)
+        C, n = esp.espace_calib_read(h, K)
+        assert n == nseq
+        if normalized:
+            # the library rounds the unit-norm rows to bf16 before the tensor-core products
+            terms = [oracle.nl_mse_term(_unit_rows_bf16(Xi), _unit_rows_bf16(Gi)) for Xi, Gi in zip(Xs, Gs)]
+        else:
+            terms = [oracle.nl_mse_term(f64(Xi), f64(Gi)) for Xi, Gi in zip(Xs, Gs)]
+        C_o = sum(terms) / nseq
+        err = np.linalg.norm(C - C_o) / np.linalg.norm(C_o)
+        assert err <= 1e-4, err
+        with pytest.raises(esp.EspaceError):
+            esp.espace_calib_accumulate(h, dev(Xs[0]))          # kinds do not mix
+        p = esp.espace_build_projection(h, dev(W), L)
+        w = esp.espace_proj_eigenvalues(p)
+        w_o, V_o, _ = oracle.eigh(C_o)
+        w_o, V_o = oracle.order_eigenpairs(w_o, V_o)
+        scale = np.abs(w_o).max()
+        if w_o[-1] < 0:
+            assert np.all(np.diff(np.abs(w)) <= 1e-12 * scale)
+        assert np.allclose(np.sort(w), np.sort(w_o), rtol=0, atol=2e-4 * scale)
+        P_o = oracle.normalize_signs(V_o[:, :L])
+        Pb = synth.bf16_to_f64(torch.from_numpy(esp.espace_proj_read_P(p).view(np.int16)).view(torch.bfloat16))
+        gap = abs(w_o[L - 1]) - abs(w_o[L])
+        proj = np.linalg.norm(Pb @ Pb.T - P_o @ P_o.T, 2)
+        assert proj <= 2e-4 * np.linalg.norm(C_o) / gap + 2e-2, (proj, gap)
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Y)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        assert_y_close(Y, oracle.forward(f64(X), Pb, f64(W))[0])
+    finally:
+        if p:
+            esp.espace_proj_destroy(p)
+        esp.espace_calib_destroy(h)
+
+
 # ------------------------------------------------------------------ tensor-parallel ranks (Sec. B.2)
 
 TP_CASES = [

@@ -437,3 +437,94 @@ def test_tp_row_projections_are_optimal_per_rank():
     Pc, _, wc = oracle.build_projection_tp(S, n, L, "column", tp)
     P1, _, w1, _ = oracle.build_projection(S, n, L)
     assert all(np.array_equal(Pc[q], P1) for q in range(tp)) and np.allclose(wc[0], w1)
+
+
+# ---------------------------------------------------------------- NL-MSE (Thm. 2, App. A.4)
+
+def test_nl_mse_term_brute_force():
+    """C_i = (X^T X G^T G + G^T G X^T X) / T^2 from the definition, pure-Python loops."""
+    r = rng(31)
+    T, K = 3, 4
+    X, G = r.standard_normal((T, K)), r.standard_normal((T, K))
+    C = oracle.nl_mse_term(X, G)
+    A = [[sum(X[t][p] * X[t][q] for t in range(T)) for q in range(K)] for p in range(K)]
+    B = [[sum(G[t][p] * G[t][q] for t in range(T)) for q in range(K)] for p in range(K)]
+    for p in range(K):
+        for q in range(K):
+            ref = sum(A[p][s] * B[s][q] + B[p][s] * A[s][q] for s in range(K)) / T ** 2
+            assert abs(C[p, q] - ref) < 1e-12
+
+
+def test_nl_mse_single_token_quadratic_form():
+    """One token (T = 1): p^T C p = 2 (x.g)(p.x)(p.g), and over an orthonormal set the sum is
+    2 <g, x> <g, P P^T x>, the term App. A.4 maximizes (the NL-MSE bound of Prop. 1)."""
+    r = rng(32)
+    K, L = 7, 3
+    x, g = r.standard_normal(K), r.standard_normal(K)
+    C = oracle.nl_mse_term(x[None, :], g[None, :])
+    for _ in range(5):
+        p = r.standard_normal(K)
+        assert abs(p @ C @ p - 2 * (x @ g) * (p @ x) * (p @ g)) < 1e-10 * (1 + abs(p @ C @ p))
+    P = synth.haar_orthonormal(r, K, L)
+    lhs = sum(P[:, l] @ C @ P[:, l] for l in range(L))
+    assert abs(lhs - 2 * (g @ x) * (g @ (P @ (P.T @ x)))) < 1e-10
+
+
+def test_nl_mse_trace_is_twice_the_cross_gram_norm():
+    """tr((A B + B A) / T^2) = 2 ||G X^T||_F^2 / T^2 (token-pair dot products)."""
+    r = rng(33)
+    T, K = 9, 6
+    X, G = r.standard_normal((T, K)), r.standard_normal((T, K))
+    C = oracle.nl_mse_term(X, G)
+    cross = sum((G[s] @ X[t]) ** 2 for s in range(T) for t in range(T))
+    assert abs(np.trace(C) - 2 * cross / T ** 2) < 1e-10 * cross
+
+
+def test_nl_mse_with_gradients_equal_to_activations_is_mse_squared():
+    """G = X: C = 2 C_X^2 with C_X = X^T X / T, so its eigenvectors are Thm. 1's and its
+    eigenvalues 2 lambda^2 (the order of C_X's eigenvalues is kept: all are positive)."""
+    r = rng(34)
+    T, K, L = 40, 6, 3
+    X = r.standard_normal((T, K)) @ np.diag(np.linspace(2.0, 0.3, K))
+    C = oracle.nl_mse_term(X, X)
+    w, V, _ = oracle.eigh(C)
+    P1, _, w1, _ = oracle.build_projection(oracle.autocorr_sum(X), T, L)
+    assert np.allclose(w, 2 * w1 ** 2, rtol=1e-10)
+    assert np.allclose(V[:, :L] @ V[:, :L].T, P1 @ P1.T, atol=1e-9)
+
+
+def test_nl_mse_normalized_is_scale_invariant_per_row():
+    r = rng(35)
+    T, K = 8, 5
+    X, G = r.standard_normal((T, K)), r.standard_normal((T, K))
+    sx, sg = np.exp(r.standard_normal((T, 1))), np.exp(r.standard_normal((T, 1)))
+    C = oracle.nl_mse_term(X, G, normalized=True)
+    assert np.allclose(oracle.nl_mse_term(X * sx, G * sg, normalized=True), C, atol=1e-12)
+    Xz = X.copy()
+    Xz[2] = 0.0
+    Cz = oracle.nl_mse_term(Xz, G, normalized=True)
+    Xd = np.delete(X, 2, axis=0)
+    Xd = Xd / np.linalg.norm(Xd, axis=1, keepdims=True)
+    Gn = G / np.linalg.norm(G, axis=1, keepdims=True)
+    A = Xd.T @ Xd
+    B = Gn.T @ Gn
+    assert np.allclose(Cz, (A @ B + B @ A) / T ** 2, atol=1e-12)
+
+
+def test_eigenpair_order_by_magnitude_only_when_indefinite():
+    """Activations and gradients with opposite anisotropy (G's strong directions rotated
+    onto X's weak ones) give an indefinite C: magnitude order, C = V diag(w) V^T kept. A
+    positive semidefinite C keeps the decreasing order."""
+    r = rng(36)
+    X = r.standard_normal((30, 6)) @ np.diag([4, 2, 1, 0.5, 0.2, 0.1])
+    G = r.standard_normal((30, 6)) @ np.diag([0.1, 0.2, 0.5, 1, 2, 4]) @ synth.haar_orthonormal(r, 6, 6).T
+    C = oracle.nl_mse_term(X, G)
+    w, V, _ = oracle.eigh(C)
+    assert w[-1] < -1e-3 * np.abs(w).max()          # indefinite
+    wo, Vo = oracle.order_eigenpairs(w, V)
+    assert np.all(np.diff(np.abs(wo)) <= 1e-15 * np.abs(wo).max())
+    assert np.allclose(Vo @ np.diag(wo) @ Vo.T, C, atol=1e-12 * np.abs(w).max())
+    Cp = oracle.nl_mse_term(X, X)                    # positive semidefinite
+    wp, Vp, _ = oracle.eigh(Cp)
+    wq, Vq = oracle.order_eigenpairs(wp, Vp)
+    assert np.array_equal(wq, wp) and np.array_equal(Vq, Vp)
