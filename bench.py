@@ -580,7 +580,28 @@ def config_rows(esp, peak_tc, peak_hbm):
     layer["total"]["speedup"] = layer["total"]["dense_ms"] / layer["total"]["espace_ms"]
     rows["llama2_layer_prefill_batch1_seq4096"] = layer
     rows["table2_tp_folded_gemm_latency"] = table2_rows(esp, peak_tc)
+    rows["nl_mse_calibration"] = nl_mse_row(esp, peak_tc, seed)
     return rows
+
+
+def nl_mse_row(esp, peak_tc, seed, K=4096, T=4096, reps=4):
+    """Thm. 2's NL-MSE calibration at K = 4096, one sequence of 4096 tokens per call with
+    synthetic gradients (an independent token model, scaled down): per call two SYRKs of T
+    tokens (2 T K (K+1) flop) and six upper-triangle K x K x K products for A B + B A with
+    bf16 hi / lo halves (6 K^2 (K+1) flop)."""
+    X = synth.ActivationModel(K, seed=seed).sample_device(T, stream="calib_tokens")
+    G = (synth.ActivationModel(K, seed=seed + 1, outliers=0, lognormal_sigma=0.0)
+         .sample_device(T, stream="calib_tokens", chunk=1).float() * 0.01).to(torch.bfloat16)
+    h = esp.espace_calib_create(K)
+    try:
+        esp.espace_calib_accumulate_nl(h, X, G)          # allocates the handle's scratch
+        ms = events_ms(lambda i: esp.espace_calib_accumulate_nl(h, X, G), reps=reps, warm=1)
+        esp.espace_check()
+    finally:
+        esp.espace_calib_destroy(h)
+    flops = 2.0 * T * K * (K + 1) + 6.0 * K * K * (K + 1)
+    return {"K": K, "tokens_per_sequence": T, "ms_per_sequence": ms, "tflops": flops / ms / 1e9,
+            "frac_tensor_peak": flops / ms / 1e9 / peak_tc}
 
 
 def graph_time_us(call, per_graph=20, replays=10):
