@@ -175,6 +175,37 @@ int espace_proj_import(int64_t K, int64_t M, int64_t L, const uint16_t* PT_host,
 void espace_proj_destroy(espace_proj_t p);
 
 /* ---------------------------------------------------------------------------------------
+ * Training view (Sec. 2.2): during training or fine-tuning the layer is
+ * Y = W^T (P P^T X) with P static and W trainable. In token-major storage the order that
+ * saves work is Z = X P (kept for the backward pass: N x L instead of N x K), Y = Z (W P)^T,
+ * with W' = P^T W refolded after every weight update. All calls below are asynchronous on
+ * the caller's stream and need a plain (not tensor-parallel) handle (ESPACE_ERR_STATE).
+ * ------------------------------------------------------------------------------------- */
+
+/* W'^T = W P_b again, rounded to bf16, from new weights W_dev ([M][K] bf16). */
+int espace_proj_refold(espace_proj_t p, const void* W_dev, void* stream);
+
+/* Z_dev ([N][Lp] bf16, caller-owned; Lp = L rounded up to 64, columns >= L come out zero)
+ * = bf16(X P_b) and Y_dev ([N][M] bf16) = bf16(Z W'), the products of
+ * espace_linear_forward with Z written where the caller keeps it. */
+int espace_train_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Z_dev, void* Y_dev,
+                         void* stream);
+
+/* The backward pass of the training view for the output gradient dY_dev ([N][M] bf16) and
+ * the Z_dev of the forward pass: dX_dev ([N][K] bf16) = bf16(bf16(dY W'^T) P_b^T), the
+ * gradient with respect to the input (through P P^T), and dW_dev ([M][K] fp32, overwritten)
+ * = bf16(dY^T Z) P_b^T, the gradient with respect to W: 2 L (2 N M + N K + M K) flop
+ * against the dense layer's 4 N M K. Scratch on the handle: N Lp + 6 Lp M bytes (the
+ * first call with a larger N grows it synchronously). */
+int espace_train_backward(espace_proj_t p, const void* dY_dev, const void* Z_dev, int64_t N,
+                          void* dX_dev, float* dW_dev, void* stream);
+
+/* The dense layer's backward pass (Eq. 1): dX_dev ([N][K] bf16) = bf16(dY W) and dW_dev
+ * ([M][K] fp32, overwritten) = dY^T X, for dY_dev [N][M], X_dev [N][K], W_dev [M][K]. */
+int espace_dense_backward(const void* dY_dev, int64_t N, const void* X_dev, int64_t K,
+                          const void* W_dev, int64_t M, void* dX_dev, float* dW_dev, void* stream);
+
+/* ---------------------------------------------------------------------------------------
  * Tensor-parallel layers folded onto one GPU (Sec. B.2, Table 2; latency method of Sec. B.4)
  *
  * Under tensor parallelism the paper applies ESPACE per rank, each rank r of tp with its

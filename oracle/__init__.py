@@ -21,6 +21,8 @@ arrays and chains the steps in the order the paper states them:
   principal eigenvectors (ordered by |eigenvalue|, as the paper does when C is indefinite);
 * ``forward_tp`` / ``build_projection_tp``  ESPACE applied per tensor-parallel rank
   (Sec. B.2, Table 2), the ranks folded onto one device (Sec. B.4);
+* ``train_backward`` / ``dense_backward``  the training view of Sec. 2.2, Y = W^T (P P^T X)
+  with P static: gradients with respect to X and W, in the order that keeps Z;
 * ``nl_mse_term`` / ``order_eigenpairs``  Thm. 2's NL-MSE matrix for one calibration
   sequence (App. A.4's per-sequence form) and the eigenvalue order the paper uses when a
   calibrated C is not positive definite.
@@ -319,3 +321,26 @@ def order_eigenpairs(w, V, tol: float = 1e-6):
         order = np.argsort(-np.abs(w), kind="stable")
         return w[order], V[:, order]
     return w, V
+
+
+def train_backward(dY, Z, P_b, Wf, round_bf16: bool = True):
+    """Backward pass of the training view (Sec. 2.2): the layer is ``Y = W^T (P P^T X)``,
+    computed as ``Z = P^T X`` and ``Y = W'^T Z`` with ``W' = P^T W`` (Eq. 3's associativity),
+    P static. For the output gradient ``dY`` ([N, M]), the saved ``Z`` ([N, L]), ``P_b``
+    ([K, L]) and ``Wf`` = W' ([L, M]):
+    ``dZ = dY W'^T`` (bf16), ``dX = dZ P^T`` (bf16) -- the input gradient passes through the
+    projection P P^T -- and ``dW = (dY^T Z) P^T`` with ``dY^T Z`` rounded to bf16 (fp64 result).
+    Returns ``(dX [N, K], dW [M, K])``."""
+    dY, Z, P_b, Wf = _f64(dY), _f64(Z), _f64(P_b), _f64(Wf)
+    rnd = bf16_round if round_bf16 else (lambda a: a)
+    dZ = rnd(dY @ Wf.T)
+    dX = rnd(dZ @ P_b.T)
+    dWP = rnd(dY.T @ Z)
+    return dX, dWP @ P_b.T
+
+
+def dense_backward(dY, X, W):
+    """Backward pass of Eq. 1, ``Y = W^T X`` stored as ``Y = X W^T``: ``dX = dY W`` and
+    ``dW = dY^T X`` (fp64). Returns ``(dX [N, K], dW [M, K])``."""
+    dY, X, W = _f64(dY), _f64(X), _f64(W)
+    return dY @ W, dY.T @ X

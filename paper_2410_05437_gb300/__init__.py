@@ -34,7 +34,8 @@ __all__ = [
     "espace_host_eigh",
     "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "PATH_TENSOR_SPLIT", "EXPORTED_SYMBOLS",
     "TP_COLUMN", "TP_ROW", "espace_proj_tp_from_host", "espace_build_projection_tp", "espace_proj_tp_info",
-    "espace_calib_accumulate_nl",
+    "espace_calib_accumulate_nl", "espace_proj_refold", "espace_train_forward", "espace_train_backward",
+    "espace_dense_backward",
     "espace_linear_forward_launches",
 ]
 
@@ -99,6 +100,10 @@ _SIGNATURES = {
     "espace_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_linear_forward_launches": (ctypes.c_int, [_vp, _i64, ctypes.c_int]),
     "espace_dense_forward": (ctypes.c_int, [_vp, _i64, _i64, _vp, _i64, _vp, _vp]),
+    "espace_proj_refold": (ctypes.c_int, [_vp, _vp, _vp]),
+    "espace_train_forward": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp, _vp]),
+    "espace_train_backward": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _vp, _vp]),
+    "espace_dense_backward": (ctypes.c_int, [_vp, _i64, _vp, _i64, _vp, _i64, _vp, _vp, _vp]),
     "espace_check": (ctypes.c_int, [_vp]),
     "espace_debug_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _vp]),
     "espace_set_wait_limit_ns": (ctypes.c_int, [ctypes.c_uint64]),
@@ -375,3 +380,24 @@ def espace_dense_forward(X, W, Y, stream=None) -> None:
     N, K = X.shape
     M = W.shape[0]
     _check(lib.espace_dense_forward(_dev_ptr(X), N, K, _dev_ptr(W), M, _dev_ptr(Y), _stream(stream)))
+
+
+def espace_proj_refold(p: int, W, stream=None) -> None:
+    _check(lib.espace_proj_refold(p, _dev_ptr(W), _stream(stream)))
+
+
+def espace_train_forward(p: int, X, Z, Y, stream=None) -> None:
+    """X [N][K], Z [N][Lp] (kept for the backward pass), Y [N][M]: device bf16."""
+    _check(lib.espace_train_forward(p, _dev_ptr(X), int(X.shape[0]), _dev_ptr(Z), _dev_ptr(Y), _stream(stream)))
+
+
+def espace_train_backward(p: int, dY, Z, dX, dW, stream=None) -> None:
+    """dY [N][M], Z [N][Lp], dX [N][K] device bf16; dW [M][K] device fp32 (overwritten)."""
+    _check(lib.espace_train_backward(p, _dev_ptr(dY), _dev_ptr(Z), int(dY.shape[0]), _dev_ptr(dX),
+                                     _dev_ptr(dW, "float32"), _stream(stream)))
+
+
+def espace_dense_backward(dY, X, W, dX, dW, stream=None) -> None:
+    """dY [N][M], X [N][K], W [M][K], dX [N][K] device bf16; dW [M][K] device fp32."""
+    _check(lib.espace_dense_backward(_dev_ptr(dY), int(dY.shape[0]), _dev_ptr(X), int(X.shape[1]), _dev_ptr(W),
+                                     int(W.shape[0]), _dev_ptr(dX), _dev_ptr(dW, "float32"), _stream(stream)))

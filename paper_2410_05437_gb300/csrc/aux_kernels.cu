@@ -98,6 +98,21 @@ cudaError_t launch_sym_split_bf16(const float* Su, int64_t K, float scale, void*
     return cudaGetLastError();
 }
 
+__global__ void f32_to_bf16_kernel(const float* __restrict__ src, int64_t count, __nv_bfloat16* __restrict__ dst)
+{
+    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < count;
+         e += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        dst[e] = __float2bfloat16_rn(src[e]);
+}
+
+cudaError_t launch_f32_to_bf16(const float* src, int64_t count, void* dst, cudaStream_t stream)
+{
+    if (count <= 0) return cudaSuccess;
+    const int64_t blocks = std::min<int64_t>((count + 255) / 256, 65536);
+    f32_to_bf16_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(src, count, static_cast<__nv_bfloat16*>(dst));
+    return cudaGetLastError();
+}
+
 // T = A B for K x K row-major fp64 matrices: 64 x 64 output tiles, 256 threads with 4 x 4
 // outputs each, 16-deep slices of A and B staged in shared memory; each output summed in
 // k order.

@@ -195,6 +195,11 @@ struct espace_proj_s {
     // r M/tp ..). ROW: PT is [tp L][K/tp], WfT is [M][tp L] (rank r's in columns r L ..).
     int tp = 1;
     int tp_kind = 0;
+    // training view: backward scratch, grown on demand
+    uint16_t* dz = nullptr;        // [dz_cap][Lp] bf16: dY W'^T
+    int64_t dz_cap = 0;
+    float* dwp32 = nullptr;        // [Lp][M] fp32: Z^T dY
+    uint16_t* dwp16 = nullptr;     // [Lp][M] bf16
     std::mutex mu;                 // guards scratch growth
 };
 
@@ -907,6 +912,9 @@ void espace_proj_destroy(espace_proj_t p)
     if (p->bar) cudaFree(p->bar);
     if (p->ready) cudaFree(p->ready);
     if (p->part) cudaFree(p->part);
+    if (p->dz) cudaFree(p->dz);
+    if (p->dwp32) cudaFree(p->dwp32);
+    if (p->dwp16) cudaFree(p->dwp16);
     delete p;
 }
 
@@ -1134,6 +1142,119 @@ int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_
     CUDA_TRY(launch_gemm_tn(X_dev, K, W_dev, K, static_cast<int>(N), static_cast<int>(M), static_cast<int>(K), Y_dev, M,
                             static_cast<cudaStream_t>(stream)),
              "espace_dense_forward: launch");
+    return ESPACE_OK;
+}
+
+// ---------------------------------------------------------------------------- training view
+
+int espace_proj_refold(espace_proj_t p, const void* W_dev, void* stream)
+{
+    if (p == nullptr || W_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_proj_refold: null pointer");
+    if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "espace_proj_refold: tensor-parallel handle");
+    if (!aligned16(W_dev)) return fail(ESPACE_ERR_ALIGN, "espace_proj_refold: W not 16-byte aligned");
+    DeviceGuard g(p->device);
+    CUDA_TRY(launch_gemm_tn(W_dev, p->K, p->PT, p->K, static_cast<int>(p->M), static_cast<int>(p->Lp),
+                            static_cast<int>(p->K), p->WfT, p->Lp, static_cast<cudaStream_t>(stream)),
+             "espace_proj_refold: launch");
+    return ESPACE_OK;
+}
+
+static int train_check(espace_proj_t p, int64_t N, const char* what)
+{
+    if (p == nullptr) return fail(ESPACE_ERR_ARG, "%s: null handle", what);
+    if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "%s: tensor-parallel handle", what);
+    if (N < 0 || N > (int64_t(1) << 31) - 256) return fail(ESPACE_ERR_SHAPE, "%s: N=%lld", what, (long long)N);
+    return ESPACE_OK;
+}
+
+int espace_train_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Z_dev, void* Y_dev, void* stream)
+{
+    int rc = train_check(p, N, "espace_train_forward");
+    if (rc != ESPACE_OK || N == 0) return rc;
+    if (X_dev == nullptr || Z_dev == nullptr || Y_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_train_forward: null pointer");
+    if (!aligned16(X_dev) || !aligned16(Z_dev) || !aligned16(Y_dev))
+        return fail(ESPACE_ERR_ALIGN, "espace_train_forward: pointers must be 16-byte aligned");
+    DeviceGuard g(p->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    rc = ensure_z(p, N, st);   // the fused launch's readiness counters
+    if (rc != ESPACE_OK) return rc;
+    const int n = static_cast<int>(N), K = static_cast<int>(p->K), M = static_cast<int>(p->M), Lp = static_cast<int>(p->Lp);
+    if (fused_forward_applies(n, Lp, M)) {
+        CUDA_TRY(launch_forward_fused(X_dev, p->PT, Z_dev, p->WfT, Y_dev, n, K, Lp, M, p->ready,
+                                      p->ready + (p->zcap + 255) / 256, st),
+                 "espace_train_forward: fused kernel");
+    } else {
+        CUDA_TRY(launch_gemm_tn(X_dev, K, p->PT, K, n, Lp, K, Z_dev, Lp, st), "espace_train_forward: Z");
+        CUDA_TRY(launch_gemm_tn(Z_dev, Lp, p->WfT, Lp, n, M, Lp, Y_dev, M, st), "espace_train_forward: Y");
+    }
+    return ESPACE_OK;
+}
+
+int espace_train_backward(espace_proj_t p, const void* dY_dev, const void* Z_dev, int64_t N, void* dX_dev,
+                          float* dW_dev, void* stream)
+{
+    int rc = train_check(p, N, "espace_train_backward");
+    if (rc != ESPACE_OK) return rc;
+    if (dW_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_train_backward: null pointer");
+    if (N > 0 && (dY_dev == nullptr || Z_dev == nullptr || dX_dev == nullptr))
+        return fail(ESPACE_ERR_ARG, "espace_train_backward: null pointer");
+    if ((N > 0 && (!aligned16(dY_dev) || !aligned16(Z_dev) || !aligned16(dX_dev))) || !aligned16(dW_dev))
+        return fail(ESPACE_ERR_ALIGN, "espace_train_backward: pointers must be 16-byte aligned");
+    DeviceGuard g(p->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t K = p->K, M = p->M, Lp = p->Lp;
+    {
+        std::lock_guard<std::mutex> lock(p->mu);
+        if (p->dwp32 == nullptr) {
+            cudaError_t e = cudaMalloc(&p->dwp32, sizeof(float) * Lp * M);
+            if (e == cudaSuccess) e = cudaMalloc(&p->dwp16, sizeof(uint16_t) * Lp * M);
+            if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_train_backward: scratch: %s", cudaGetErrorString(e));
+        }
+        if (p->dz_cap < N) {
+            CUDA_TRY(cudaStreamSynchronize(st), "espace_train_backward: sync before scratch growth");
+            if (p->dz) cudaFree(p->dz);
+            p->dz = nullptr;
+            p->dz_cap = 0;
+            cudaError_t e = cudaMalloc(&p->dz, sizeof(uint16_t) * N * Lp);
+            if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_train_backward: scratch: %s", cudaGetErrorString(e));
+            p->dz_cap = N;
+        }
+    }
+    CUDA_TRY(launch_zero_f32(dW_dev, K * M, st), "espace_train_backward: clear dW");
+    if (N == 0) return ESPACE_OK;
+    const int n = static_cast<int>(N), k = static_cast<int>(K), m = static_cast<int>(M), lp = static_cast<int>(Lp);
+    // dZ = dY W' (W' = P^T W: W'^T is [M][Lp], read M/N-major)
+    CUDA_TRY(launch_gemm_nn(dY_dev, M, p->WfT, Lp, n, lp, m, p->dz, Lp, st), "espace_train_backward: dZ");
+    // dX = dZ P^T (P^T is [Lp][K], read M/N-major)
+    CUDA_TRY(launch_gemm_nn(p->dz, Lp, p->PT, K, n, k, lp, dX_dev, K, st), "espace_train_backward: dX");
+    // (dW P)^T = Z^T dY over the tokens, then dW = (dW P) P^T over the rank index
+    CUDA_TRY(launch_zero_f32(p->dwp32, Lp * M, st), "espace_train_backward: clear");
+    CUDA_TRY(launch_gemm_tn_tokens_f32(Z_dev, lp, dY_dev, m, N, p->dwp32, M, st), "espace_train_backward: Z^T dY");
+    CUDA_TRY(launch_f32_to_bf16(p->dwp32, Lp * M, p->dwp16, st), "espace_train_backward: round");
+    CUDA_TRY(launch_gemm_tn_tokens_f32(p->dwp16, m, p->PT, k, Lp, dW_dev, K, st), "espace_train_backward: dW");
+    return ESPACE_OK;
+}
+
+int espace_dense_backward(const void* dY_dev, int64_t N, const void* X_dev, int64_t K, const void* W_dev, int64_t M,
+                          void* dX_dev, float* dW_dev, void* stream)
+{
+    if (N < 0) return fail(ESPACE_ERR_SHAPE, "espace_dense_backward: N < 0");
+    if (dW_dev == nullptr || W_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_dense_backward: null pointer");
+    if (N > 0 && (dY_dev == nullptr || X_dev == nullptr || dX_dev == nullptr))
+        return fail(ESPACE_ERR_ARG, "espace_dense_backward: null pointer");
+    if (K < 8 || K % 8 != 0 || K > 65536 || M < 8 || M % 8 != 0 || M > (int64_t(1) << 30) || N > (int64_t(1) << 31) - 256)
+        return fail(ESPACE_ERR_SHAPE, "espace_dense_backward: unsupported shape N=%lld K=%lld M=%lld", (long long)N, (long long)K,
+                    (long long)M);
+    if ((N > 0 && (!aligned16(dY_dev) || !aligned16(X_dev) || !aligned16(dX_dev))) || !aligned16(W_dev) || !aligned16(dW_dev))
+        return fail(ESPACE_ERR_ALIGN, "espace_dense_backward: pointers must be 16-byte aligned");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    CUDA_TRY(launch_zero_f32(dW_dev, K * M, st), "espace_dense_backward: clear dW");
+    if (N == 0) return ESPACE_OK;
+    // dX = dY W (W [M][K] read M/N-major), dW = dY^T X over the tokens
+    CUDA_TRY(launch_gemm_nn(dY_dev, M, W_dev, K, static_cast<int>(N), static_cast<int>(K), static_cast<int>(M), dX_dev, K, st),
+             "espace_dense_backward: dX");
+    CUDA_TRY(launch_gemm_tn_tokens_f32(dY_dev, static_cast<int>(M), X_dev, static_cast<int>(K), N, dW_dev, K, st),
+             "espace_dense_backward: dW");
     return ESPACE_OK;
 }
 

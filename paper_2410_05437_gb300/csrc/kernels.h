@@ -60,6 +60,17 @@ cudaError_t launch_gemm_tn_blocks(const void* A, int64_t lda, int a_cols, const 
                                   const int* ak0, const int* c0, const int* cw, int kdim, void* C, int64_t ldc,
                                   cudaStream_t stream);
 
+// C[rows][cols] (bf16, leading dimension ldc) = A[rows][kdim] B[kdim][cols] with B stored
+// row-major (its columns contiguous: an M/N-major tcgen05 operand), on CTA pairs; A and B
+// bf16 with leading dimensions lda, ldb (multiples of 8).
+cudaError_t launch_gemm_nn(const void* A, int64_t lda, const void* B, int64_t ldb, int rows, int cols, int kdim,
+                           void* C, int64_t ldc, cudaStream_t stream);
+// out[R][C] (fp32, leading dimension ldo) += U^T V for token-major U[N][R], V[N][C] (bf16,
+// rows contiguous): a reduction over tokens, as for weight gradients; atomics, so out is
+// zeroed by the caller for a plain product. R and C multiples of 8.
+cudaError_t launch_gemm_tn_tokens_f32(const void* U, int R, const void* V, int C, int64_t N, float* out,
+                                     int64_t ldo, cudaStream_t stream);
+
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
 // The same kernel with two operands: S's upper triangle += that of X^T Y (X, Y [N][K] bf16).
@@ -99,6 +110,9 @@ cudaError_t launch_sym_full_f64(const float* Su, int64_t K, double scale, double
 cudaError_t launch_sym_split_bf16(const float* Su, int64_t K, float scale, void* hi, void* lo, cudaStream_t stream);
 // T = A B for K x K row-major fp64 matrices.
 cudaError_t launch_gemm_f64(const double* A, const double* B, int K, double* T, cudaStream_t stream);
+
+// dst[i] = bf16(src[i]) (round to nearest even).
+cudaError_t launch_f32_to_bf16(const float* src, int64_t count, void* dst, cudaStream_t stream);
 
 // Fills dst[count] with zeros (fp32).
 cudaError_t launch_zero_f32(float* dst, int64_t count, cudaStream_t stream);

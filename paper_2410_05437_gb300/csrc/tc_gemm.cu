@@ -364,6 +364,7 @@ struct PairProblem {
     const int2* tile_list;   // (tile row, tile col) pairs, or nullptr for the full grid
     void* out;
     int64_t ldo;
+    int upper;               // token-reduction (M/N-major) programs: add only column >= row
 };
 
 // A program of one product, or of two where the second one's A operand is the first one's
@@ -441,6 +442,7 @@ __device__ __forceinline__ PairProblem pair_problem_of(const PairArgs& a, int pr
     r.tile_list = prob == 0 ? a.p[0].tile_list : a.p[1].tile_list;
     r.out = prob == 0 ? a.p[0].out : a.p[1].out;
     r.ldo = prob == 0 ? a.p[0].ldo : a.p[1].ldo;
+    r.upper = prob == 0 ? a.p[0].upper : a.p[1].upper;
     return r;
 }
 
@@ -491,11 +493,13 @@ __device__ __forceinline__ void fence_proxy_async_global()
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-// SYRK = false: K-major operands, bf16 stores (the products of Eq. 3 and Eq. 1).
-// SYRK = true: both operands are one token-major X read M/N-major (64 features x 64 tokens
-// per box, two boxes per operand and CTA), and the epilogue adds each tile's upper triangle
-// (column >= row) to the fp32 sum S with atomics (Eq. 4).
-template <bool SYRK>
+// SYRK = false: K-major A, bf16 stores (the products of Eq. 3 and Eq. 1); B K-major, or with
+// B_MN M/N-major (B stored [k][cols], e.g. the weights of a backward product dY W).
+// SYRK = true: both operands are token-major matrices read M/N-major (64 features x 64
+// tokens per box, two boxes per operand and CTA): C = U^T V reduces over tokens, and the
+// epilogue adds each tile (its upper triangle, column >= row, when the problem says so) to
+// an fp32 sum with atomics (Eq. 4; weight gradients).
+template <bool SYRK, bool B_MN = SYRK>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THREADS, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_b0,
                         const __grid_constant__ CUtensorMap map_a1, const __grid_constant__ CUtensorMap map_b1,
@@ -606,10 +610,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                         // 64 features x 64 tokens per box; the second 64 features at +8 KB
                         tma_load_2d_pair(sa, ma, bar, row_a, kb * BK);
                         tma_load_2d_pair(sa + 8192, ma, bar, row_a + 64, kb * BK);
+                    } else {
+                        tma_load_2d_pair(sa, ma, bar, ak0 + kb * BK, row_a);
+                    }
+                    if (B_MN) {
                         tma_load_2d_pair(sb, mb, bar, row_b, kb * BK);
                         tma_load_2d_pair(sb + 8192, mb, bar, row_b + 64, kb * BK);
                     } else {
-                        tma_load_2d_pair(sa, ma, bar, ak0 + kb * BK, row_a);
                         tma_load_2d_pair(sb, mb, bar, kb * BK, row_b);
                     }
                     if (++stage == PAIR_STAGES) {
@@ -623,11 +630,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer (leader)
         if (lane == 0 && leader) {
-            constexpr uint32_t idesc = idesc_bf16_f32(PAIR_BM, PAIR_BN, SYRK, SYRK);
+            static_assert(!SYRK || B_MN, "token-reduction programs read both operands M/N-major");
+            constexpr uint32_t idesc = idesc_bf16_f32(PAIR_BM, PAIR_BN, SYRK, B_MN);
             // K-major: the next 16-element K slice starts 32 bytes along the swizzled row;
             // M/N-major: 16 tokens further = 16 rows of 128 bytes, 64-feature atoms 8 KB apart
-            constexpr uint32_t k_step = SYRK ? 2048u : 32u;
-            constexpr uint32_t lbo = SYRK ? 8192u : 16u;
+            constexpr uint32_t a_step = SYRK ? 2048u : 32u, a_lbo = SYRK ? 8192u : 16u;
+            constexpr uint32_t b_step = B_MN ? 2048u : 32u, b_lbo = B_MN ? 8192u : 16u;
             int stage = 0;
             uint32_t phase = 0;
             int acc = 0;
@@ -658,8 +666,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                         const uint32_t b_addr = a_addr + PAIR_A_BYTES;
 #pragma unroll
                         for (int j = 0; j < BK / UMMA_K; ++j) {
-                            const uint64_t ad = smem_desc_sw128(a_addr + j * k_step, lbo, 1024);
-                            const uint64_t bd = smem_desc_sw128(b_addr + j * k_step, lbo, 1024);
+                            const uint64_t ad = smem_desc_sw128(a_addr + j * a_step, a_lbo, 1024);
+                            const uint64_t bd = smem_desc_sw128(b_addr + j * b_step, b_lbo, 1024);
                             umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > c0 || j > 0) ? 1u : 0u);
                         }
                         umma_commit_pair(&empty[stage], 0x3);   // frees the stage in both CTAs
@@ -722,21 +730,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                 }
             }
             if (!ok) break;
-            // S[row][col] += run for the upper triangle (col >= row), 16 bytes at a time
+            // S[row][col] += run (for col >= row only when the problem is a triangle), 16
+            // bytes at a time
             const int row = tm * PAIR_BM + row_in_tile;
             if (row < pb.rows) {
                 float* s_row = reinterpret_cast<float*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
                 const int colb = tn * PAIR_BN + half * 128;
+                const int cmin = pb.upper ? row : 0;
 #pragma unroll
                 for (int i = 0; i < 128; i += 4) {
                     const int col = colb + i;
-                    if (col >= row && col + 3 < pb.cols) {
+                    if (col >= cmin && col + 3 < pb.cols) {
                         atomicAdd(reinterpret_cast<float4*>(s_row + col),
                                   make_float4(run[i], run[i + 1], run[i + 2], run[i + 3]));
                     } else {
 #pragma unroll
                         for (int j = 0; j < 4; ++j)
-                            if (col + j >= row && col + j < pb.cols) atomicAdd(s_row + col + j, run[i + j]);
+                            if (col + j >= cmin && col + j < pb.cols) atomicAdd(s_row + col + j, run[i + j]);
                     }
                 }
             }
@@ -892,12 +902,12 @@ PairProblem pair_problem(int rows, int cols, int kdim, void* out, int64_t ldo)
     return p;
 }
 
-template <bool SYRK>
+template <bool SYRK, bool B_MN = SYRK>
 cudaError_t launch_pair(const CUtensorMap* maps, PairArgs& a, const DeviceInfo* dev, cudaStream_t stream)
 {
     const int items = a.p[0].num_tiles * a.p[0].ksplit + (a.nprob > 1 ? a.p[1].num_tiles * a.p[1].ksplit : 0);
     const int pairs = std::min(items, dev->num_sms / 2);
-    auto kern = tc_gemm_pair_kernel<SYRK>;
+    auto kern = tc_gemm_pair_kernel<SYRK, B_MN>;
     static bool attr_set[64] = {};
     if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
     if (!attr_set[dev->device]) {
@@ -1210,6 +1220,7 @@ cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int
         p.tile_list = tiles;
         p.out = S;
         p.ldo = K;
+        p.upper = 1;
         a.nprob = 1;
         a.status = dev->status;
         a.wait_limit_ns = wait_limit_ns();
@@ -1238,6 +1249,56 @@ cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int
     a.wait_limit_ns = wait_limit_ns();
     const int grid = std::min(a.num_tiles * a.ksplit, dev->num_sms);
     return launch_kernel<256, 4, true, EPI_ATOMIC_UPPER_F32>(mx, my, a, grid, stream);
+}
+
+cudaError_t launch_gemm_tn_tokens_f32(const void* U, int R, const void* V, int C, int64_t N, float* out,
+                                     int64_t ldo, cudaStream_t stream)
+{
+    if (N <= 0 || R <= 0 || C <= 0) return cudaSuccess;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    if (dev->num_sms < 2) return cudaErrorInvalidConfiguration;
+    CUtensorMap maps[4];
+    if (!encode_map(&maps[0], U, R, static_cast<uint64_t>(N), R, 64, BK)) return cudaErrorInvalidValue;
+    if (!encode_map(&maps[1], V, C, static_cast<uint64_t>(N), C, 64, BK)) return cudaErrorInvalidValue;
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+    PairArgs a{};
+    PairProblem& p = a.p[0];
+    p.rows = R;
+    p.cols = C;
+    p.kblocks = static_cast<int>((N + BK - 1) / BK);
+    p.tiles_n = (C + PAIR_BN - 1) / PAIR_BN;
+    p.num_tiles = ((R + PAIR_BM - 1) / PAIR_BM) * p.tiles_n;
+    choose_splits(p.kblocks, p.num_tiles, dev->num_sms / 2, &p.ksplit, &p.kb_per_split);
+    p.tile_list = nullptr;
+    p.out = out;
+    p.ldo = ldo;
+    p.upper = 0;
+    a.nprob = 1;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return launch_pair<true>(maps, a, dev, stream);
+}
+
+cudaError_t launch_gemm_nn(const void* A, int64_t lda, const void* B, int64_t ldb, int rows, int cols, int kdim,
+                           void* C, int64_t ldc, cudaStream_t stream)
+{
+    if (rows <= 0 || cols <= 0) return cudaSuccess;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    if (dev->num_sms < 2) return cudaErrorInvalidConfiguration;
+    CUtensorMap maps[4];
+    if (!encode_map(&maps[0], A, kdim, rows, lda, BK, 128)) return cudaErrorInvalidValue;
+    if (!encode_map(&maps[1], B, cols, kdim, ldb, 64, BK)) return cudaErrorInvalidValue;
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+    PairArgs a{};
+    a.p[0] = pair_problem(rows, cols, kdim, C, ldc);
+    a.nprob = 1;
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return launch_pair<false, true>(maps, a, dev, stream);
 }
 
 cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,

@@ -291,6 +291,81 @@ def test_single_token_forward_repeated_and_interleaved(esp):
         esp.espace_proj_destroy(p)
 
 
+# ------------------------------------------------------------------ training view (Sec. 2.2)
+
+def assert_close_normwise(A_gpu, A_ref, rel=Y_REL, mx_rel=Y_MAX):
+    A = f64(A_gpu) if A_gpu.dtype == torch.bfloat16 else A_gpu.double().cpu().numpy()
+    err = np.linalg.norm(A - A_ref) / max(np.linalg.norm(A_ref), 1e-300)
+    mx = np.abs(A - A_ref).max() / max(np.abs(A_ref).max(), 1e-300)
+    assert np.all(np.isfinite(A))
+    assert err <= rel, f"normwise error {err:.3e}"
+    assert mx <= mx_rel, f"max error {mx:.3e}"
+
+
+TRAIN_CASES = [
+    # (N, K, M, L)
+    (300, 512, 776, 256),      # two launches forward, ragged M
+    (1000, 1024, 1000, 512),   # fused forward, ragged N and M
+    (129, 520, 264, 100),      # ragged K and L (Z padded to 128 columns)
+    (2048, 1024, 2048, 512),   # several tiles each way
+]
+
+
+@pytest.mark.parametrize("N,K,M,L", TRAIN_CASES)
+def test_train_forward_backward_matches_oracle(esp, N, K, M, L):
+    """Y = W^T (P P^T X) with P static: the forward keeps Z, the backward returns dX (through
+    P P^T) and dW = (dY^T Z) P^T, each against the oracle; then a weight update refolds W'."""
+    seed = 4000 + N + K
+    _, X, W = make_layer(K, M, N, seed=seed)
+    P = synth.random_projection(K, L, seed=seed)
+    r = np.random.default_rng(seed)
+    dY = torch.from_numpy(r.standard_normal((N, M)).astype(np.float32)).to(torch.bfloat16)
+    Lp = (L + 63) // 64 * 64
+    p = esp.espace_proj_from_host(P, dev(W))
+    try:
+        Z = torch.full((N, Lp), float("nan"), dtype=torch.bfloat16, device="cuda")
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_train_forward(p, dev(X), Z, Y)
+        dX = torch.full((N, K), float("nan"), dtype=torch.bfloat16, device="cuda")
+        dW = torch.full((M, K), float("nan"), dtype=torch.float32, device="cuda")
+        esp.espace_train_backward(p, dev(dY), Z, dX, dW)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        Pb = oracle.bf16_round(P)
+        Wf = oracle.fold(Pb, f64(W))
+        Y_o, Z_o, _ = oracle.forward(f64(X), Pb, f64(W), Wf=Wf)
+        Zg = f64(Z)
+        assert np.all(Zg[:, L:] == 0)
+        assert_close_normwise(Z[:, :L], Z_o)
+        assert_y_close(Y, Y_o)
+        dX_o, dW_o = oracle.train_backward(f64(dY), Zg[:, :L], Pb, Wf)
+        assert_close_normwise(dX, dX_o)
+        assert_close_normwise(dW, dW_o)
+        # an optimizer step: new weights, W' refolded on the device
+        W2 = synth.weights(M, K, seed=seed + 1)
+        esp.espace_proj_refold(p, dev(W2))
+        esp.espace_train_forward(p, dev(X), Z, Y)
+        torch.cuda.synchronize()
+        assert_y_close(Y, oracle.forward(f64(X), Pb, f64(W2))[0])
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+@pytest.mark.parametrize("N,K,M", [(300, 512, 776), (2048, 1024, 2048), (129, 136, 392)])
+def test_dense_backward_matches_oracle(esp, N, K, M):
+    _, X, W = make_layer(K, M, N, seed=5000 + N)
+    r = np.random.default_rng(N)
+    dY = torch.from_numpy(r.standard_normal((N, M)).astype(np.float32)).to(torch.bfloat16)
+    dX = torch.empty((N, K), dtype=torch.bfloat16, device="cuda")
+    dW = torch.empty((M, K), dtype=torch.float32, device="cuda")
+    esp.espace_dense_backward(dev(dY), dev(X), dev(W), dX, dW)
+    torch.cuda.synchronize()
+    esp.espace_check()
+    dX_o, dW_o = oracle.dense_backward(f64(dY), f64(X), f64(W))
+    assert_close_normwise(dX, dX_o)
+    assert_close_normwise(dW, dW_o, rel=1e-5, mx_rel=1e-4)
+
+
 # ------------------------------------------------------------------ NL-MSE calibration (Thm. 2)
 
 def _unit_rows_bf16(A):

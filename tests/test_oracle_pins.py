@@ -528,3 +528,62 @@ def test_eigenpair_order_by_magnitude_only_when_indefinite():
     wp, Vp, _ = oracle.eigh(Cp)
     wq, Vq = oracle.order_eigenpairs(wp, Vp)
     assert np.array_equal(wq, wp) and np.array_equal(Vq, Vp)
+
+
+# ---------------------------------------------------------------- training view (Sec. 2.2)
+
+def _train_loss(X, W, P, R):
+    """sum(R * Y) for Y = W^T (P P^T X), token-major: Y = X P P^T W^T."""
+    return float(np.sum(R * (X @ P @ P.T @ W.T)))
+
+
+def test_train_backward_matches_finite_differences():
+    """Unrounded gradients of sum(R * Y) against central differences of the forward."""
+    r = rng(41)
+    N, K, M, L = 4, 6, 5, 3
+    X, W, R = r.standard_normal((N, K)), r.standard_normal((M, K)), r.standard_normal((N, M))
+    P = synth.haar_orthonormal(r, K, L)
+    Z = oracle.project(X, P, round_bf16=False)
+    dX, dW = oracle.train_backward(R, Z, P, oracle.fold(P, W, round_bf16=False), round_bf16=False)
+    h = 1e-6
+    for (i, j) in ((0, 0), (1, 3), (3, 5), (2, 2)):
+        Xp, Xm = X.copy(), X.copy()
+        Xp[i, j] += h
+        Xm[i, j] -= h
+        fd = (_train_loss(Xp, W, P, R) - _train_loss(Xm, W, P, R)) / (2 * h)
+        assert abs(dX[i, j] - fd) < 1e-7 * (1 + abs(fd))
+    for (m, k) in ((0, 0), (4, 5), (2, 3)):
+        Wp, Wm = W.copy(), W.copy()
+        Wp[m, k] += h
+        Wm[m, k] -= h
+        fd = (_train_loss(X, Wp, P, R) - _train_loss(X, Wm, P, R)) / (2 * h)
+        assert abs(dW[m, k] - fd) < 1e-7 * (1 + abs(fd))
+
+
+def test_train_backward_full_rank_is_the_dense_backward():
+    """P = I (L = K): the training view is the dense layer, and so are its gradients."""
+    r = rng(42)
+    N, K, M = 5, 7, 6
+    X, W, dY = r.standard_normal((N, K)), r.standard_normal((M, K)), r.standard_normal((N, M))
+    P = np.eye(K)
+    dX, dW = oracle.train_backward(dY, X, P, oracle.fold(P, W, round_bf16=False), round_bf16=False)
+    dXd, dWd = oracle.dense_backward(dY, X, W)
+    for t in range(N):
+        for k in range(K):
+            assert abs(dXd[t, k] - sum(dY[t][m] * W[m][k] for m in range(M))) < 1e-12
+    for m in range(M):
+        for k in range(K):
+            assert abs(dWd[m, k] - sum(dY[t][m] * X[t][k] for t in range(N))) < 1e-12
+    assert np.allclose(dX, dXd, atol=1e-12) and np.allclose(dW, dWd, atol=1e-12)
+
+
+def test_train_input_gradient_is_the_adjoint():
+    """<dY, J V> = <J^T dY, V> for the map X -> X P P^T W^T (linear in X)."""
+    r = rng(43)
+    N, K, M, L = 6, 9, 4, 4
+    W, dY, V = r.standard_normal((M, K)), r.standard_normal((N, M)), r.standard_normal((N, K))
+    P = synth.haar_orthonormal(r, K, L)
+    Wf = oracle.fold(P, W, round_bf16=False)
+    JV = oracle.forward(V, P, W, Wf=Wf, round_bf16=False)[0]
+    dX, _ = oracle.train_backward(dY, oracle.project(V, P, round_bf16=False), P, Wf, round_bf16=False)
+    assert abs(np.sum(dY * JV) - np.sum(dX * V)) < 1e-10 * (1 + abs(np.sum(dY * JV)))
