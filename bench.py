@@ -581,27 +581,58 @@ def config_rows(esp, peak_tc, peak_hbm):
     rows["llama2_layer_prefill_batch1_seq4096"] = layer
     rows["table2_tp_folded_gemm_latency"] = table2_rows(esp, peak_tc)
     rows["nl_mse_calibration"] = nl_mse_row(esp, peak_tc, seed)
+    rows["training_step"] = training_rows(esp, peak_tc, seed)
     return rows
 
 
-def nl_mse_row(esp, peak_tc, seed, K=4096, T=4096, reps=4):
-    """Thm. 2's NL-MSE calibration at K = 4096, one sequence of 4096 tokens per call with
-    synthetic gradients (an independent token model, scaled down): per call two SYRKs of T
-    tokens (2 T K (K+1) flop) and six upper-triangle K x K x K products for A B + B A with
-    bf16 hi / lo halves (6 K^2 (K+1) flop)."""
-    X = synth.ActivationModel(K, seed=seed).sample_device(T, stream="calib_tokens")
-    G = (synth.ActivationModel(K, seed=seed + 1, outliers=0, lognormal_sigma=0.0)
-         .sample_device(T, stream="calib_tokens", chunk=1).float() * 0.01).to(torch.bfloat16)
-    h = esp.espace_calib_create(K)
-    try:
-        esp.espace_calib_accumulate_nl(h, X, G)          # allocates the handle's scratch
-        ms = events_ms(lambda i: esp.espace_calib_accumulate_nl(h, X, G), reps=reps, warm=1)
-        esp.espace_check()
-    finally:
-        esp.espace_calib_destroy(h)
-    flops = 2.0 * T * K * (K + 1) + 6.0 * K * K * (K + 1)
-    return {"K": K, "tokens_per_sequence": T, "ms_per_sequence": ms, "tflops": flops / ms / 1e9,
-            "frac_tensor_peak": flops / ms / 1e9 / peak_tc}
+def training_rows(esp, peak_tc, seed, micro=4):
+    """The training view of Sec. 2.2 against dense training, one layer's GEMM work per
+    optimizer step of `micro` micro-batches: ESPACE refolds W' = P^T W once (after the
+    weight update), runs each micro-batch's forward (keeping Z) and backward (dX, and Z^T dY
+    accumulated), then forms dW = (sum Z^T dY)^T P^T once; dense runs each micro-batch's
+    forward and backward (dX, dW accumulated). Llama2-7B QKV (4096 -> 12288) with 4096-token
+    micro-batches, L = K/2 and Table 2's L = 1024; GPT3-22B FC1 (6144 -> 24576) with
+    2048-token micro-batches, L = 2048."""
+    out = {}
+    for name, K, M, L, N in (("llama2_qkv_L2048", 4096, 12288, 2048, 4096), ("llama2_qkv_L1024", 4096, 12288, 1024, 4096),
+                             ("gpt3_22b_fc1_L2048", 6144, 24576, 2048, 2048)):
+        W = synth.weights_device(M, K, seed=seed)
+        X = synth.ActivationModel(K, seed=seed).sample_device(N)
+        dY = (torch.randn((N, M), device="cuda") * 0.01).to(torch.bfloat16)
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        dX = torch.empty((N, K), dtype=torch.bfloat16, device="cuda")
+        dW = torch.empty((M, K), dtype=torch.float32, device="cuda")
+        Lp = (L + 63) // 64 * 64
+        Z = torch.empty((N, Lp), dtype=torch.bfloat16, device="cuda")
+        p = device_projection(esp, K, L, W, seed)
+
+        def espace_step(i):
+            esp.espace_proj_refold(p, W)
+            for _ in range(micro):
+                esp.espace_train_forward(p, X, Z, Y)
+                esp.espace_train_backward(p, dY, Z, dX)
+            esp.espace_train_weight_grad(p, dW)
+
+        def dense_step(i):
+            for j in range(micro):
+                esp.espace_dense_forward(X, W, Y)
+                esp.espace_dense_backward(dY, X, W, dX, dW, accumulate=j > 0)
+
+        try:
+            e_ms = events_ms(espace_step)
+            d_ms = events_ms(dense_step)
+            esp.espace_check()
+        finally:
+            esp.espace_proj_destroy(p)
+        T = micro * N
+        eflops = 2.0 * M * K * L + 2.0 * T * L * (K + M) + 2.0 * T * L * (2 * M + K) + 2.0 * L * M * K
+        dflops = 6.0 * T * K * M
+        out[name] = {"K": K, "M": M, "L": L, "tokens_per_micro_batch": N, "micro_batches": micro,
+                     "espace_step_ms": e_ms, "dense_step_ms": d_ms, "step_speedup": d_ms / e_ms,
+                     "espace_flops_over_dense": eflops / dflops, "espace_tflops": eflops / e_ms / 1e9,
+                     "espace_frac_tensor_peak": eflops / e_ms / 1e9 / peak_tc, "dense_tflops": dflops / d_ms / 1e9}
+        del W, X, dY, Y, dX, dW, Z
+    return out
 
 
 def graph_time_us(call, per_graph=20, replays=10):

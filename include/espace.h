@@ -191,19 +191,26 @@ int espace_proj_refold(espace_proj_t p, const void* W_dev, void* stream);
 int espace_train_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Z_dev, void* Y_dev,
                          void* stream);
 
-/* The backward pass of the training view for the output gradient dY_dev ([N][M] bf16) and
- * the Z_dev of the forward pass: dX_dev ([N][K] bf16) = bf16(bf16(dY W'^T) P_b^T), the
- * gradient with respect to the input (through P P^T), and dW_dev ([M][K] fp32, overwritten)
- * = bf16(dY^T Z) P_b^T, the gradient with respect to W: 2 L (2 N M + N K + M K) flop
- * against the dense layer's 4 N M K. Scratch on the handle: N Lp + 6 Lp M bytes (the
+/* The backward pass of the training view for one micro-batch: for the output gradient
+ * dY_dev ([N][M] bf16) and the Z_dev of its forward pass, dX_dev ([N][K] bf16) =
+ * bf16(bf16(dY W'^T) P_b^T), the gradient with respect to the input (through P P^T), and
+ * (dW P)^T += Z^T dY into an fp32 accumulator of the handle ([Lp][M]): 2 L N (2 M + K)
+ * flop against the dense layer's 4 N M K. Scratch on the handle: N Lp + 6 Lp M bytes (the
  * first call with a larger N grows it synchronously). */
 int espace_train_backward(espace_proj_t p, const void* dY_dev, const void* Z_dev, int64_t N,
-                          void* dX_dev, float* dW_dev, void* stream);
+                          void* dX_dev, void* stream);
+
+/* At the end of a step (after the micro-batches' backward passes): dW_dev ([M][K] fp32,
+ * overwritten) = bf16(sum of dY^T Z) P_b^T, the gradient with respect to W (2 L M K flop,
+ * once per step), and the accumulator is cleared for the next step. */
+int espace_train_weight_grad(espace_proj_t p, float* dW_dev, void* stream);
 
 /* The dense layer's backward pass (Eq. 1): dX_dev ([N][K] bf16) = bf16(dY W) and dW_dev
- * ([M][K] fp32, overwritten) = dY^T X, for dY_dev [N][M], X_dev [N][K], W_dev [M][K]. */
+ * ([M][K] fp32) = dY^T X, or dW_dev += dY^T X when accumulate != 0 (micro-batches of one
+ * step), for dY_dev [N][M], X_dev [N][K], W_dev [M][K]. */
 int espace_dense_backward(const void* dY_dev, int64_t N, const void* X_dev, int64_t K,
-                          const void* W_dev, int64_t M, void* dX_dev, float* dW_dev, void* stream);
+                          const void* W_dev, int64_t M, void* dX_dev, float* dW_dev, int accumulate,
+                          void* stream);
 
 /* ---------------------------------------------------------------------------------------
  * Tensor-parallel layers folded onto one GPU (Sec. B.2, Table 2; latency method of Sec. B.4)

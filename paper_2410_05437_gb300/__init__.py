@@ -35,6 +35,7 @@ __all__ = [
     "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "PATH_TENSOR_SPLIT", "EXPORTED_SYMBOLS",
     "TP_COLUMN", "TP_ROW", "espace_proj_tp_from_host", "espace_build_projection_tp", "espace_proj_tp_info",
     "espace_calib_accumulate_nl", "espace_proj_refold", "espace_train_forward", "espace_train_backward",
+    "espace_train_weight_grad",
     "espace_dense_backward",
     "espace_linear_forward_launches",
 ]
@@ -102,8 +103,9 @@ _SIGNATURES = {
     "espace_dense_forward": (ctypes.c_int, [_vp, _i64, _i64, _vp, _i64, _vp, _vp]),
     "espace_proj_refold": (ctypes.c_int, [_vp, _vp, _vp]),
     "espace_train_forward": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp, _vp]),
-    "espace_train_backward": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _vp, _vp]),
-    "espace_dense_backward": (ctypes.c_int, [_vp, _i64, _vp, _i64, _vp, _i64, _vp, _vp, _vp]),
+    "espace_train_backward": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _vp]),
+    "espace_train_weight_grad": (ctypes.c_int, [_vp, _vp, _vp]),
+    "espace_dense_backward": (ctypes.c_int, [_vp, _i64, _vp, _i64, _vp, _i64, _vp, _vp, ctypes.c_int, _vp]),
     "espace_check": (ctypes.c_int, [_vp]),
     "espace_debug_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _vp]),
     "espace_set_wait_limit_ns": (ctypes.c_int, [ctypes.c_uint64]),
@@ -391,13 +393,20 @@ def espace_train_forward(p: int, X, Z, Y, stream=None) -> None:
     _check(lib.espace_train_forward(p, _dev_ptr(X), int(X.shape[0]), _dev_ptr(Z), _dev_ptr(Y), _stream(stream)))
 
 
-def espace_train_backward(p: int, dY, Z, dX, dW, stream=None) -> None:
-    """dY [N][M], Z [N][Lp], dX [N][K] device bf16; dW [M][K] device fp32 (overwritten)."""
-    _check(lib.espace_train_backward(p, _dev_ptr(dY), _dev_ptr(Z), int(dY.shape[0]), _dev_ptr(dX),
-                                     _dev_ptr(dW, "float32"), _stream(stream)))
+def espace_train_backward(p: int, dY, Z, dX, stream=None) -> None:
+    """dY [N][M], Z [N][Lp], dX [N][K] device bf16; the weight gradient accumulates on the
+    handle until espace_train_weight_grad."""
+    _check(lib.espace_train_backward(p, _dev_ptr(dY), _dev_ptr(Z), int(dY.shape[0]), _dev_ptr(dX), _stream(stream)))
 
 
-def espace_dense_backward(dY, X, W, dX, dW, stream=None) -> None:
-    """dY [N][M], X [N][K], W [M][K], dX [N][K] device bf16; dW [M][K] device fp32."""
+def espace_train_weight_grad(p: int, dW, stream=None) -> None:
+    """dW [M][K] device fp32 (overwritten): the step's weight gradient."""
+    _check(lib.espace_train_weight_grad(p, _dev_ptr(dW, "float32"), _stream(stream)))
+
+
+def espace_dense_backward(dY, X, W, dX, dW, accumulate: bool = False, stream=None) -> None:
+    """dY [N][M], X [N][K], W [M][K], dX [N][K] device bf16; dW [M][K] device fp32
+    (overwritten, or added to with accumulate)."""
     _check(lib.espace_dense_backward(_dev_ptr(dY), int(dY.shape[0]), _dev_ptr(X), int(X.shape[1]), _dev_ptr(W),
-                                     int(W.shape[0]), _dev_ptr(dX), _dev_ptr(dW, "float32"), _stream(stream)))
+                                     int(W.shape[0]), _dev_ptr(dX), _dev_ptr(dW, "float32"), int(bool(accumulate)),
+                                     _stream(stream)))

@@ -1159,6 +1159,25 @@ int espace_proj_refold(espace_proj_t p, const void* W_dev, void* stream)
     return ESPACE_OK;
 }
 
+// The fp32 accumulator of (dW P)^T ([Lp][M], zeroed) and its bf16 copy, made on first use.
+static int ensure_grad_acc(espace_proj_s* p, cudaStream_t st)
+{
+    std::lock_guard<std::mutex> lock(p->mu);
+    if (p->dwp32 != nullptr) return ESPACE_OK;
+    const int64_t count = p->Lp * p->M;
+    cudaError_t e = cudaMalloc(&p->dwp32, sizeof(float) * count);
+    if (e == cudaSuccess) e = cudaMalloc(&p->dwp16, sizeof(uint16_t) * count);
+    if (e == cudaSuccess) e = launch_zero_f32(p->dwp32, count, st);
+    if (e != cudaSuccess) {
+        if (p->dwp32) cudaFree(p->dwp32);
+        if (p->dwp16) cudaFree(p->dwp16);
+        p->dwp32 = nullptr;
+        p->dwp16 = nullptr;
+        return fail(ESPACE_ERR_NOMEM, "training view: gradient accumulator: %s", cudaGetErrorString(e));
+    }
+    return ESPACE_OK;
+}
+
 static int train_check(espace_proj_t p, int64_t N, const char* what)
 {
     if (p == nullptr) return fail(ESPACE_ERR_ARG, "%s: null handle", what);
@@ -1191,25 +1210,21 @@ int espace_train_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Z_
 }
 
 int espace_train_backward(espace_proj_t p, const void* dY_dev, const void* Z_dev, int64_t N, void* dX_dev,
-                          float* dW_dev, void* stream)
+                          void* stream)
 {
     int rc = train_check(p, N, "espace_train_backward");
-    if (rc != ESPACE_OK) return rc;
-    if (dW_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_train_backward: null pointer");
-    if (N > 0 && (dY_dev == nullptr || Z_dev == nullptr || dX_dev == nullptr))
+    if (rc != ESPACE_OK || N == 0) return rc;
+    if (dY_dev == nullptr || Z_dev == nullptr || dX_dev == nullptr)
         return fail(ESPACE_ERR_ARG, "espace_train_backward: null pointer");
-    if ((N > 0 && (!aligned16(dY_dev) || !aligned16(Z_dev) || !aligned16(dX_dev))) || !aligned16(dW_dev))
+    if (!aligned16(dY_dev) || !aligned16(Z_dev) || !aligned16(dX_dev))
         return fail(ESPACE_ERR_ALIGN, "espace_train_backward: pointers must be 16-byte aligned");
     DeviceGuard g(p->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int64_t K = p->K, M = p->M, Lp = p->Lp;
+    rc = ensure_grad_acc(p, st);
+    if (rc != ESPACE_OK) return rc;
     {
         std::lock_guard<std::mutex> lock(p->mu);
-        if (p->dwp32 == nullptr) {
-            cudaError_t e = cudaMalloc(&p->dwp32, sizeof(float) * Lp * M);
-            if (e == cudaSuccess) e = cudaMalloc(&p->dwp16, sizeof(uint16_t) * Lp * M);
-            if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_train_backward: scratch: %s", cudaGetErrorString(e));
-        }
         if (p->dz_cap < N) {
             CUDA_TRY(cudaStreamSynchronize(st), "espace_train_backward: sync before scratch growth");
             if (p->dz) cudaFree(p->dz);
@@ -1220,23 +1235,38 @@ int espace_train_backward(espace_proj_t p, const void* dY_dev, const void* Z_dev
             p->dz_cap = N;
         }
     }
-    CUDA_TRY(launch_zero_f32(dW_dev, K * M, st), "espace_train_backward: clear dW");
-    if (N == 0) return ESPACE_OK;
     const int n = static_cast<int>(N), k = static_cast<int>(K), m = static_cast<int>(M), lp = static_cast<int>(Lp);
     // dZ = dY W' (W' = P^T W: W'^T is [M][Lp], read M/N-major)
     CUDA_TRY(launch_gemm_nn(dY_dev, M, p->WfT, Lp, n, lp, m, p->dz, Lp, st), "espace_train_backward: dZ");
     // dX = dZ P^T (P^T is [Lp][K], read M/N-major)
     CUDA_TRY(launch_gemm_nn(p->dz, Lp, p->PT, K, n, k, lp, dX_dev, K, st), "espace_train_backward: dX");
-    // (dW P)^T = Z^T dY over the tokens, then dW = (dW P) P^T over the rank index
-    CUDA_TRY(launch_zero_f32(p->dwp32, Lp * M, st), "espace_train_backward: clear");
+    // (dW P)^T += Z^T dY over the tokens (the weight gradient waits for the step's end)
     CUDA_TRY(launch_gemm_tn_tokens_f32(Z_dev, lp, dY_dev, m, N, p->dwp32, M, st), "espace_train_backward: Z^T dY");
-    CUDA_TRY(launch_f32_to_bf16(p->dwp32, Lp * M, p->dwp16, st), "espace_train_backward: round");
-    CUDA_TRY(launch_gemm_tn_tokens_f32(p->dwp16, m, p->PT, k, Lp, dW_dev, K, st), "espace_train_backward: dW");
+    return ESPACE_OK;
+}
+
+int espace_train_weight_grad(espace_proj_t p, float* dW_dev, void* stream)
+{
+    int rc = train_check(p, 0, "espace_train_weight_grad");
+    if (rc != ESPACE_OK) return rc;
+    if (dW_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_train_weight_grad: null pointer");
+    if (!aligned16(dW_dev)) return fail(ESPACE_ERR_ALIGN, "espace_train_weight_grad: dW not 16-byte aligned");
+    DeviceGuard g(p->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t K = p->K, M = p->M, Lp = p->Lp;
+    rc = ensure_grad_acc(p, st);
+    if (rc != ESPACE_OK) return rc;
+    // dW = (dW P) P^T: the accumulated (dW P)^T rounded to bf16, reduced over the rank index
+    CUDA_TRY(launch_f32_to_bf16(p->dwp32, Lp * M, p->dwp16, st), "espace_train_weight_grad: round");
+    CUDA_TRY(launch_zero_f32(dW_dev, K * M, st), "espace_train_weight_grad: clear dW");
+    CUDA_TRY(launch_gemm_tn_tokens_f32(p->dwp16, static_cast<int>(M), p->PT, static_cast<int>(K), Lp, dW_dev, K, st),
+             "espace_train_weight_grad: dW");
+    CUDA_TRY(launch_zero_f32(p->dwp32, Lp * M, st), "espace_train_weight_grad: reset");
     return ESPACE_OK;
 }
 
 int espace_dense_backward(const void* dY_dev, int64_t N, const void* X_dev, int64_t K, const void* W_dev, int64_t M,
-                          void* dX_dev, float* dW_dev, void* stream)
+                          void* dX_dev, float* dW_dev, int accumulate, void* stream)
 {
     if (N < 0) return fail(ESPACE_ERR_SHAPE, "espace_dense_backward: N < 0");
     if (dW_dev == nullptr || W_dev == nullptr) return fail(ESPACE_ERR_ARG, "espace_dense_backward: null pointer");
@@ -1248,7 +1278,7 @@ int espace_dense_backward(const void* dY_dev, int64_t N, const void* X_dev, int6
     if ((N > 0 && (!aligned16(dY_dev) || !aligned16(X_dev) || !aligned16(dX_dev))) || !aligned16(W_dev) || !aligned16(dW_dev))
         return fail(ESPACE_ERR_ALIGN, "espace_dense_backward: pointers must be 16-byte aligned");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    CUDA_TRY(launch_zero_f32(dW_dev, K * M, st), "espace_dense_backward: clear dW");
+    if (!accumulate) CUDA_TRY(launch_zero_f32(dW_dev, K * M, st), "espace_dense_backward: clear dW");
     if (N == 0) return ESPACE_OK;
     // dX = dY W (W [M][K] read M/N-major), dW = dY^T X over the tokens
     CUDA_TRY(launch_gemm_nn(dY_dev, M, W_dev, K, static_cast<int>(N), static_cast<int>(K), static_cast<int>(M), dX_dev, K, st),

@@ -328,7 +328,8 @@ def test_train_forward_backward_matches_oracle(esp, N, K, M, L):
         esp.espace_train_forward(p, dev(X), Z, Y)
         dX = torch.full((N, K), float("nan"), dtype=torch.bfloat16, device="cuda")
         dW = torch.full((M, K), float("nan"), dtype=torch.float32, device="cuda")
-        esp.espace_train_backward(p, dev(dY), Z, dX, dW)
+        esp.espace_train_backward(p, dev(dY), Z, dX)
+        esp.espace_train_weight_grad(p, dW)
         torch.cuda.synchronize()
         esp.espace_check()
         Pb = oracle.bf16_round(P)
@@ -341,6 +342,18 @@ def test_train_forward_backward_matches_oracle(esp, N, K, M, L):
         dX_o, dW_o = oracle.train_backward(f64(dY), Zg[:, :L], Pb, Wf)
         assert_close_normwise(dX, dX_o)
         assert_close_normwise(dW, dW_o)
+        # two micro-batches of one step: the weight gradient sums over both (their tokens)
+        X2 = make_layer(K, M, N, seed=seed + 2)[1]
+        dY2 = torch.from_numpy(r.standard_normal((N, M)).astype(np.float32)).to(torch.bfloat16)
+        Z2 = torch.empty_like(Z)
+        esp.espace_train_forward(p, dev(X2), Z2, Y)
+        esp.espace_train_backward(p, dev(dY), Z, dX)
+        esp.espace_train_backward(p, dev(dY2), Z2, dX)
+        esp.espace_train_weight_grad(p, dW)
+        torch.cuda.synchronize()
+        both = np.concatenate([Zg[:, :L], f64(Z2)[:, :L]])
+        _, dW_o2 = oracle.train_backward(np.concatenate([f64(dY), f64(dY2)]), both, Pb, Wf)
+        assert_close_normwise(dW, dW_o2)
         # an optimizer step: new weights, W' refolded on the device
         W2 = synth.weights(M, K, seed=seed + 1)
         esp.espace_proj_refold(p, dev(W2))
@@ -364,6 +377,9 @@ def test_dense_backward_matches_oracle(esp, N, K, M):
     dX_o, dW_o = oracle.dense_backward(f64(dY), f64(X), f64(W))
     assert_close_normwise(dX, dX_o)
     assert_close_normwise(dW, dW_o, rel=1e-5, mx_rel=1e-4)
+    esp.espace_dense_backward(dev(dY), dev(X), dev(W), dX, dW, accumulate=True)
+    torch.cuda.synchronize()
+    assert_close_normwise(dW, 2 * dW_o, rel=1e-5, mx_rel=1e-4)
 
 
 # ------------------------------------------------------------------ NL-MSE calibration (Thm. 2)
