@@ -52,7 +52,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-rows", action="store_true", help="skip the side measurements")
-    ap.add_argument("--profile-case", choices=["fused", "syrk", "decode"],
+    ap.add_argument("--profile-case", choices=["fused", "syrk", "decode", "train"],
                     help="run a few launches of one kernel on a small fixed case (for ncu) and exit")
     return ap.parse_args()
 
@@ -585,6 +585,26 @@ def config_rows(esp, peak_tc, peak_hbm):
     return rows
 
 
+def nl_mse_row(esp, peak_tc, seed, K=4096, T=4096, reps=4):
+    """Thm. 2's NL-MSE calibration at K = 4096, one sequence of 4096 tokens per call with
+    synthetic gradients (an independent token model, scaled down): per call two SYRKs of T
+    tokens (2 T K (K+1) flop) and six upper-triangle K x K x K products for A B + B A with
+    bf16 hi / lo halves (6 K^2 (K+1) flop)."""
+    X = synth.ActivationModel(K, seed=seed).sample_device(T, stream="calib_tokens")
+    G = (synth.ActivationModel(K, seed=seed + 1, outliers=0, lognormal_sigma=0.0)
+         .sample_device(T, stream="calib_tokens", chunk=1).float() * 0.01).to(torch.bfloat16)
+    h = esp.espace_calib_create(K)
+    try:
+        esp.espace_calib_accumulate_nl(h, X, G)          # allocates the handle's scratch
+        ms = events_ms(lambda i: esp.espace_calib_accumulate_nl(h, X, G), reps=reps, warm=1)
+        esp.espace_check()
+    finally:
+        esp.espace_calib_destroy(h)
+    flops = 2.0 * T * K * (K + 1) + 6.0 * K * K * (K + 1)
+    return {"K": K, "tokens_per_sequence": T, "ms_per_sequence": ms, "tflops": flops / ms / 1e9,
+            "frac_tensor_peak": flops / ms / 1e9 / peak_tc}
+
+
 def training_rows(esp, peak_tc, seed, micro=4):
     """The training view of Sec. 2.2 against dense training, one layer's GEMM work per
     optimizer step of `micro` micro-batches: ESPACE refolds W' = P^T W once (after the
@@ -663,7 +683,8 @@ def graph_time_us(call, per_graph=20, replays=10):
 def profile_case(which):
     """A few launches of one kernel, with little else on the GPU: the target of the ncu
     captures summarized under profiles/ (launch 3 of the fused forward, launch 2 of the
-    calibration SYRK, launch 3 of the decode kernel)."""
+    calibration SYRK, launch 3 of the decode kernel, the training view's backward
+    products)."""
     import paper_2410_05437_gb300 as esp
     torch.cuda.set_device(0)
     if which in ("fused", "decode"):
@@ -675,6 +696,23 @@ def profile_case(which):
         Y = torch.empty(N, M, device="cuda", dtype=torch.bfloat16)
         for _ in range(3):
             esp.espace_linear_forward(p, X, Y)
+        torch.cuda.synchronize()
+        esp.espace_proj_destroy(p)
+    elif which == "train":
+        # pair-kernel launches: 1 fold, 2 forward (fused), 3 dZ = dY W', 4 dX = dZ P^T,
+        # 5 (dW P)^T += Z^T dY, 6 dW = (dW P) P^T
+        K, M, L, N = 4096, 12288, 2048, 4096
+        W = synth.weights_device(M, K)
+        p = esp.espace_proj_from_host(synth.random_projection(K, L), W)
+        X = synth.ActivationModel(K).sample_device(N)
+        dY = (torch.randn(N, M, device="cuda") * 0.01).to(torch.bfloat16)
+        Z = torch.empty(N, L, device="cuda", dtype=torch.bfloat16)
+        Y = torch.empty(N, M, device="cuda", dtype=torch.bfloat16)
+        dX = torch.empty(N, K, device="cuda", dtype=torch.bfloat16)
+        dW = torch.empty(M, K, device="cuda", dtype=torch.float32)
+        esp.espace_train_forward(p, X, Z, Y)
+        esp.espace_train_backward(p, dY, Z, dX)
+        esp.espace_train_weight_grad(p, dW)
         torch.cuda.synchronize()
         esp.espace_proj_destroy(p)
     else:
