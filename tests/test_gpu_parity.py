@@ -56,7 +56,7 @@ def make_layer(K, M, N, seed, outliers=None, sigma=0.5):
 
 @pytest.mark.parametrize("N,K,M", [(128, 512, 512), (200, 520, 264), (1, 64, 8), (300, 1024, 776),
                                    (129, 136, 392), (9, 136, 392), (32, 520, 264), (5, 4096, 12288),
-                                   (33, 2056, 1000), (256, 1024, 776)])
+                                   (33, 2056, 1000), (256, 1024, 776), (512, 4096, 2056), (300, 8192, 776)])
 def test_dense_forward_matches_oracle(esp, N, K, M):
     _, X, W = make_layer(K, M, N, seed=100 + N)
     Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
@@ -139,6 +139,8 @@ FORWARD_CASES = [
     (777, 2048, 1000, 256, 0),     # K >= 2 M and few Z tiles: rank-L product split over the SMs
     (300, 1040, 264, 64, 1),       # the same just above the swapped token range, ragged K
     (2304, 1152, 520, 1152, 1),    # 45 Z tiles: one persistent launch for both products
+    (512, 4096, 12288, 2048, 1),   # fused, more Y tiles than CTA pairs
+    (700, 6144, 1000, 520, 1),     # K >= 2 M: rank-L product split over the SMs, ragged N / L / M
     (300, 1024, 3000, 300, 3),
     # few tokens on tcgen05 with the weights as the 128-row operand; split reductions
     (100, 4096, 776, 2048, 1),     # both products split (16 and 7 weight tiles)
