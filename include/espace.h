@@ -291,6 +291,19 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
  * N = 0), or -1 for invalid arguments or a path that cannot take N. Host-only query. */
 int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path);
 
+/* Synchronous. The forward of espace_linear_forward for X and Y in host memory: X_host
+ * ([N][K] bf16) is copied to device staging owned by the handle, the products run on the
+ * caller's stream, and Y ([N][M] bf16) is copied back into Y_host; the call returns with
+ * Y_host filled (work already on the caller's stream runs first, and later work on it
+ * waits for the copies). N is cut into up to 8 chunks of at least 1024 tokens: the copy of
+ * chunk j + 1 in, chunk j's products and the copy of chunk j - 1 out overlap, on two
+ * streams of the handle. Pinned (page-locked) host buffers let the copies run
+ * asynchronously; pageable ones still give the right result. The first call with a larger
+ * N than any before allocates the staging (N (K + M) bf16 values). One call at a time per
+ * handle. */
+int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host,
+                               void* stream);
+
 /* Capacity, in bf16 values, of the fixed scratch used by espace_linear_forward_noalloc:
  * 16 MiB, enough for N * Lp <= 8,388,608 (e.g. 4096 tokens at L = 2048). */
 #define ESPACE_NOALLOC_Z_ELEMS 8388608

@@ -195,6 +195,12 @@ struct espace_proj_s {
     // r M/tp ..). ROW: PT is [tp L][K/tp], WfT is [M][tp L] (rank r's in columns r L ..).
     int tp = 1;
     int tp_kind = 0;
+    // host-buffer forward: device staging of X and Y, copy streams and per-chunk events
+    uint16_t* hx = nullptr;
+    uint16_t* hy = nullptr;
+    int64_t h_cap = 0;
+    cudaStream_t s_in = nullptr, s_out = nullptr;
+    cudaEvent_t ev[2 * 16 + 2] = {};
     // training view: backward scratch, grown on demand
     uint16_t* dz = nullptr;        // [dz_cap][Lp] bf16: dY W'^T
     int64_t dz_cap = 0;
@@ -915,6 +921,12 @@ void espace_proj_destroy(espace_proj_t p)
     if (p->dz) cudaFree(p->dz);
     if (p->dwp32) cudaFree(p->dwp32);
     if (p->dwp16) cudaFree(p->dwp16);
+    if (p->hx) cudaFree(p->hx);
+    if (p->hy) cudaFree(p->hy);
+    for (cudaEvent_t e : p->ev)
+        if (e) cudaEventDestroy(e);
+    if (p->s_in) cudaStreamDestroy(p->s_in);
+    if (p->s_out) cudaStreamDestroy(p->s_out);
     delete p;
 }
 
@@ -1109,6 +1121,85 @@ int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path)
 int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev, void* stream)
 {
     return espace_linear_forward_path(p, X_dev, N, Y_dev, stream, ESPACE_PATH_AUTO);
+}
+
+// Chunks of the host-buffer forward: up to 8, each at least 1024 tokens (multiples of 256),
+// so that the chunks' products stay efficient while their copies overlap.
+static int host_chunks(int64_t N, int64_t* chunk)
+{
+    int nc = static_cast<int>(std::min<int64_t>(8, std::max<int64_t>(1, N / 1024)));
+    int64_t c = (N + nc - 1) / nc;
+    c = (c + 255) / 256 * 256;
+    nc = static_cast<int>((N + c - 1) / c);
+    *chunk = c;
+    return nc;
+}
+
+int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream)
+{
+    if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward_host: null handle");
+    if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "espace_linear_forward_host: tensor-parallel handle");
+    if (N < 0 || N > (int64_t(1) << 31) - 256) return fail(ESPACE_ERR_SHAPE, "espace_linear_forward_host: N=%lld", (long long)N);
+    if (N == 0) return ESPACE_OK;
+    if (X_host == nullptr || Y_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward_host: null pointer");
+    DeviceGuard g(p->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t K = p->K, M = p->M;
+    {
+        std::lock_guard<std::mutex> lock(p->mu);
+        if (p->s_in == nullptr) {
+            cudaError_t e = cudaStreamCreateWithFlags(&p->s_in, cudaStreamNonBlocking);
+            if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p->s_out, cudaStreamNonBlocking);
+            for (cudaEvent_t& ev : p->ev)
+                if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+            if (e != cudaSuccess) return fail_cuda(e, "espace_linear_forward_host: streams");
+        }
+        if (p->h_cap < N) {
+            CUDA_TRY(cudaStreamSynchronize(st), "espace_linear_forward_host: sync before staging growth");
+            if (p->hx) cudaFree(p->hx);
+            if (p->hy) cudaFree(p->hy);
+            p->hx = p->hy = nullptr;
+            p->h_cap = 0;
+            cudaError_t e = cudaMalloc(&p->hx, sizeof(uint16_t) * N * K);
+            if (e == cudaSuccess) e = cudaMalloc(&p->hy, sizeof(uint16_t) * N * M);
+            if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_linear_forward_host: staging: %s", cudaGetErrorString(e));
+            p->h_cap = N;
+        }
+    }
+    int64_t C = 0;
+    const int nc = host_chunks(N, &C);
+    cudaEvent_t* ev_in = p->ev;           // chunk j copied in
+    cudaEvent_t* ev_done = p->ev + 16;    // chunk j computed
+    cudaEvent_t start = p->ev[32], end = p->ev[33];
+    // the copies start after the work already on the caller's stream
+    CUDA_TRY(cudaEventRecord(start, st), "espace_linear_forward_host: order");
+    CUDA_TRY(cudaStreamWaitEvent(p->s_in, start, 0), "espace_linear_forward_host: order");
+    CUDA_TRY(cudaStreamWaitEvent(p->s_out, start, 0), "espace_linear_forward_host: order");
+    const uint16_t* xh = static_cast<const uint16_t*>(X_host);
+    uint16_t* yh = static_cast<uint16_t*>(Y_host);
+    for (int j = 0; j < nc; ++j) {
+        const int64_t t0 = j * C, n = std::min(C, N - t0);
+        CUDA_TRY(cudaMemcpyAsync(p->hx + t0 * K, xh + t0 * K, sizeof(uint16_t) * n * K, cudaMemcpyHostToDevice, p->s_in),
+                 "espace_linear_forward_host: copy in");
+        CUDA_TRY(cudaEventRecord(ev_in[j], p->s_in), "espace_linear_forward_host: event");
+    }
+    for (int j = 0; j < nc; ++j) {
+        const int64_t t0 = j * C, n = std::min(C, N - t0);
+        // chunk j's product runs on the caller's stream once its tokens are on the device,
+        // while the next chunk's tokens and the previous chunk's outputs are copied
+        CUDA_TRY(cudaStreamWaitEvent(st, ev_in[j], 0), "espace_linear_forward_host: order");
+        int rc = espace_linear_forward_path(p, p->hx + t0 * K, n, p->hy + t0 * M, st, ESPACE_PATH_AUTO);
+        if (rc != ESPACE_OK) return rc;
+        CUDA_TRY(cudaEventRecord(ev_done[j], st), "espace_linear_forward_host: event");
+        CUDA_TRY(cudaStreamWaitEvent(p->s_out, ev_done[j], 0), "espace_linear_forward_host: order");
+        CUDA_TRY(cudaMemcpyAsync(yh + t0 * M, p->hy + t0 * M, sizeof(uint16_t) * n * M, cudaMemcpyDeviceToHost, p->s_out),
+                 "espace_linear_forward_host: copy out");
+    }
+    // the caller's stream continues after the last copy; the call returns with Y_host filled
+    CUDA_TRY(cudaEventRecord(end, p->s_out), "espace_linear_forward_host: event");
+    CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host: order");
+    CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host: wait");
+    return ESPACE_OK;
 }
 
 int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev, int64_t M, void* Y_dev,

@@ -224,6 +224,29 @@ def test_few_token_forward_is_reproducible(esp):
         esp.espace_proj_destroy(p)
 
 
+@pytest.mark.parametrize("N", [1, 700, 2304, 4100])
+def test_linear_forward_host_buffers(esp, N):
+    """X and Y in pinned host memory: chunks of the tokens copied in, computed and copied
+    out on overlapping streams; the result matches the device-buffer forward and the oracle."""
+    K, M, L = 1024, 1000, 512
+    _, X, W = make_layer(K, M, N, seed=6000 + N)
+    P = synth.random_projection(K, L, seed=6000 + N)
+    p = esp.espace_proj_from_host(P, dev(W))
+    try:
+        Xh = X.contiguous().pin_memory()
+        Yh = torch.full((N, M), float("nan"), dtype=torch.bfloat16).pin_memory()
+        esp.espace_linear_forward_host(p, Xh, Yh)
+        esp.espace_check()
+        assert_y_close(Yh, oracle.forward(f64(X), oracle.bf16_round(P), f64(W))[0])
+        Yd = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Yd)
+        torch.cuda.synchronize()
+        if N >= 1024:   # the same kernels on chunks of at least 1024 tokens
+            assert torch.equal(Yh.view(torch.int16), Yd.cpu().view(torch.int16))
+    finally:
+        esp.espace_proj_destroy(p)
+
+
 def test_linear_forward_full_rank_equals_dense_within_bf16(esp):
     """L = K: P P^T = I, so the projected layer reproduces the dense one (Sec. 2.2)."""
     N, K, M = 64, 256, 384
