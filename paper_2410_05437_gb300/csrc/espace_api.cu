@@ -1177,6 +1177,20 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
     CUDA_TRY(cudaStreamWaitEvent(p->s_out, start, 0), "espace_linear_forward_host: order");
     const uint16_t* xh = static_cast<const uint16_t*>(X_host);
     uint16_t* yh = static_cast<uint16_t*>(Y_host);
+    // on an error after copies were queued, wait for them before returning, so that no copy
+    // touches the caller's host buffers after the call
+    struct Drain {
+        espace_proj_s* p;
+        cudaStream_t st;
+        bool armed = true;
+        ~Drain()
+        {
+            if (!armed) return;
+            cudaStreamSynchronize(p->s_in);
+            cudaStreamSynchronize(st);
+            cudaStreamSynchronize(p->s_out);
+        }
+    } drain{p, st};
     for (int j = 0; j < nc; ++j) {
         const int64_t t0 = j * C, n = std::min(C, N - t0);
         CUDA_TRY(cudaMemcpyAsync(p->hx + t0 * K, xh + t0 * K, sizeof(uint16_t) * n * K, cudaMemcpyHostToDevice, p->s_in),
@@ -1199,6 +1213,7 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
     CUDA_TRY(cudaEventRecord(end, p->s_out), "espace_linear_forward_host: event");
     CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host: order");
     CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host: wait");
+    drain.armed = false;
     return ESPACE_OK;
 }
 
