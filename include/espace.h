@@ -295,7 +295,7 @@ int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path);
  * ([N][K] bf16) is copied to device staging owned by the handle, the products run on the
  * caller's stream, and Y ([N][M] bf16) is copied back into Y_host; the call returns with
  * Y_host filled (work already on the caller's stream runs first, and later work on it
- * waits for the copies). N is cut into up to 8 chunks of at least 1024 tokens: the copy of
+ * waits for the copies). N is cut into up to 8 chunks of at least 512 tokens: the copy of
  * chunk j + 1 in, chunk j's products and the copy of chunk j - 1 out overlap, on two
  * streams of the handle. Pinned (page-locked) host buffers let the copies run
  * asynchronously; pageable ones still give the right result. The first call with a larger
