@@ -264,6 +264,7 @@ def run_ours(args, world, rank, local):
     total_ms = max_over_ranks(t_begin.elapsed_time(t_end), world)
     phase1 = [starts[i].elapsed_time(mids[i]) for i in range(args.steps)]
     phase2 = [mids[i].elapsed_time(ends[i]) for i in range(args.steps)]
+    step_ms = [starts[i].elapsed_time(ends[i]) for i in range(args.steps)]
     ms_per_step = total_ms / args.steps
     value = flops * args.steps * world / (total_ms * 1e-3) / 1e12
     esp.espace_check()
@@ -321,6 +322,8 @@ def run_ours(args, world, rank, local):
                      "algorithmic_bytes": 2.0 * (N * K + K * L + L * M + N * M)},
         "phases_ms": {"before_event": statistics.mean(phase1), "after_event": statistics.mean(phase2),
                       "launches_per_step": 1 if fused else 2},
+        "step_ms": {"mean": statistics.mean(step_ms), "median": statistics.median(step_ms),
+                    "min": min(step_ms), "max": max(step_ms), "kernel_median": statistics.median(phase2)},
         "roofline_step": {"frac_of_tensor_peak": (flops / (ms_per_step * 1e-3) / 1e12) / peak_tc,
                           "roofline_ms": max(flops / (peak_tc * 1e12),
                                              2.0 * (N * K + K * L + L * M + N * M) / (peak_hbm * 1e9)) * 1e3},
