@@ -329,8 +329,11 @@ int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev, int64_t N,
 /* Async. The uncompressed layer of Eq. 1, Y = W^T X, as Y_dev[N][M] = X_dev[N][K] W_dev^T
  * with W_dev in [M][K] layout, with fp32 accumulation and bf16 output on the same kernel
  * families as the projected layer (N <= 8: the streaming kernel; N <= 256: tcgen05 with
- * the weights as the 128-row operand, no split; above: tcgen05): the baseline the
- * projected layer is measured against. */
+ * the weights as the 128-row operand, the reduction split over the SMs in the same cases
+ * as the projected layer's products, with fp32 partials in a per-device workspace that
+ * the first such call allocates; above: tcgen05): the baseline the projected layer is
+ * measured against. Calls that split share the device's workspace: order them on the GPU
+ * (one stream, or streams that wait on each other). */
 int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev,
                          int64_t M, void* Y_dev, void* stream);
 

@@ -1219,6 +1219,16 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
     return ESPACE_OK;
 }
 
+// Split workspace of the dense forward's few-token products, per device (dense calls on
+// one device must be ordered on the GPU: the same stream, or streams that wait on each
+// other).
+struct DenseWs {
+    float* part = nullptr;
+    int64_t cap = 0;
+    std::mutex mu;
+};
+static DenseWs g_dense_ws[64];
+
 int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev, int64_t M, void* Y_dev,
                          void* stream)
 {
@@ -1241,9 +1251,26 @@ int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_
         return ESPACE_OK;
     }
     if (N <= SWAP_MAX_TOKENS) {
-        // few tokens: the weight rows span the grid (no split: no workspace without a handle)
+        // few tokens: the weight rows span the grid, the reduction split over the SMs when
+        // the tiles would leave SMs idle (partials in the device's dense workspace)
+        float* part = nullptr;
+        const SwapPlan pl = gemm_swap_plan(static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), dev->num_sms, true);
+        if (pl.part_elems > 0 && dev->device >= 0 && dev->device < 64) {
+            DenseWs& ws = g_dense_ws[dev->device];
+            std::lock_guard<std::mutex> lock(ws.mu);
+            if (ws.cap < pl.part_elems) {
+                CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "espace_dense_forward: sync");
+                if (ws.part) cudaFree(ws.part);
+                ws.part = nullptr;
+                ws.cap = 0;
+                cudaError_t e = cudaMalloc(&ws.part, sizeof(float) * pl.part_elems);
+                if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_dense_forward: workspace: %s", cudaGetErrorString(e));
+                ws.cap = pl.part_elems;
+            }
+            part = ws.part;
+        }
         CUDA_TRY(launch_gemm_swap(W_dev, K, X_dev, K, static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), Y_dev,
-                                  M, nullptr, static_cast<cudaStream_t>(stream)),
+                                  M, part, static_cast<cudaStream_t>(stream)),
                  "espace_dense_forward: launch");
         return ESPACE_OK;
     }

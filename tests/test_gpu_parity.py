@@ -56,7 +56,7 @@ def make_layer(K, M, N, seed, outliers=None, sigma=0.5):
 
 @pytest.mark.parametrize("N,K,M", [(128, 512, 512), (200, 520, 264), (1, 64, 8), (300, 1024, 776),
                                    (129, 136, 392), (9, 136, 392), (32, 520, 264), (5, 4096, 12288),
-                                   (33, 2056, 1000), (256, 1024, 776), (512, 4096, 2056), (300, 8192, 776)])
+                                   (33, 2056, 1000), (256, 1024, 776), (512, 4096, 2056), (300, 8192, 776), (128, 4096, 12288)])
 def test_dense_forward_matches_oracle(esp, N, K, M):
     _, X, W = make_layer(K, M, N, seed=100 + N)
     Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
@@ -148,6 +148,7 @@ FORWARD_CASES = [
     (256, 2048, 1000, 1000, 0),    # 256-token tiles
     (129, 520, 264, 100, 1),       # 256-token tile, ragged
     (7, 1024, 776, 448, 1),        # fewer tokens than one MMA's rows
+    (128, 4096, 12288, 2048, 0),   # Llama2 QKV at 128 tokens
     # one token on the decode kernel, across its stage layouts
     (1, 4096, 12288, 2048, 0),     # Llama2 QKV layer
     (1, 11008, 4096, 1376, 2),     # K beyond one 2048-wide k-block, ragged
