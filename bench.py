@@ -52,7 +52,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-rows", action="store_true", help="skip the side measurements")
-    ap.add_argument("--profile-case", choices=["fused", "syrk", "decode", "train"],
+    ap.add_argument("--profile-case", choices=["fused", "syrk", "decode", "train", "nl"],
                     help="run a few launches of one kernel on a small fixed case (for ncu) and exit")
     return ap.parse_args()
 
@@ -683,7 +683,7 @@ def profile_case(which):
     """A few launches of one kernel, with little else on the GPU: the target of the ncu
     captures summarized under profiles/ (launch 3 of the fused forward, launch 2 of the
     calibration SYRK, launch 3 of the decode kernel, the training view's backward
-    products)."""
+    products, the NL-MSE launches)."""
     import paper_2410_05437_gb300 as esp
     torch.cuda.set_device(0)
     if which in ("fused", "decode"):
@@ -714,6 +714,17 @@ def profile_case(which):
         esp.espace_train_weight_grad(p, dW)
         torch.cuda.synchronize()
         esp.espace_proj_destroy(p)
+    elif which == "nl":
+        # two NL-MSE sequences of 4096 tokens at K = 4096 (11 launches each)
+        K, T = 4096, 4096
+        X = synth.ActivationModel(K).sample_device(T, stream="calib_tokens")
+        G = (synth.ActivationModel(K, seed=1, outliers=0, lognormal_sigma=0.0)
+             .sample_device(T, stream="calib_tokens", chunk=1).float() * 0.01).to(torch.bfloat16)
+        h = esp.espace_calib_create(K)
+        for _ in range(2):
+            esp.espace_calib_accumulate_nl(h, X, G)
+        torch.cuda.synchronize()
+        esp.espace_calib_destroy(h)
     else:
         K, n = 4096, 65536
         X = synth.ActivationModel(K).sample_device(n, stream="calib_tokens")

@@ -58,43 +58,101 @@ cudaError_t launch_zero_f32(float* dst, int64_t count, cudaStream_t stream)
 }
 
 // C[i][j] = scale * Su[min(i,j)][max(i,j)] (Su: fp32, upper triangle i <= j valid).
-__global__ void sym_full_f64_kernel(const float* __restrict__ Su, int64_t K, double scale, double* __restrict__ C)
+// Symmetric expansion of an upper triangle: block (tj, ti) with ti <= tj reads the 64 x 64
+// tile (ti, tj) of Su once, row by row in 16-byte pieces, and stores it together with its
+// mirror (tj, ti) through shared memory, so that every global access runs along rows; below
+// the diagonal of a diagonal tile the element comes from its transposed position.
+// store(e, v) writes output elements e .. e + 3 (e = i K + j, j a multiple of 4), whose
+// values are v[q] = S(i, j + q). K is a multiple of 4.
+template <class Store>
+__global__ void __launch_bounds__(256) sym_expand_kernel(const float* __restrict__ Su, int64_t K, Store store)
 {
-    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < K * K;
-         e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t i = e / K, j = e - i * K;
-        C[e] = scale * static_cast<double>(i <= j ? Su[i * K + j] : Su[j * K + i]);
+    __shared__ float t[64][65];
+    const int64_t ti = blockIdx.y, tj = blockIdx.x;
+    if (ti > tj) return;
+    const int64_t r0 = ti * 64, c0 = tj * 64;
+    for (int e = threadIdx.x; e < 64 * 16; e += 256) {
+        const int r = e >> 4, c = (e & 15) * 4;
+        const int64_t i = r0 + r, j = c0 + c;
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i < K && j < K) v = *reinterpret_cast<const float4*>(Su + i * K + j);
+        t[r][c] = v.x;
+        t[r][c + 1] = v.y;
+        t[r][c + 2] = v.z;
+        t[r][c + 3] = v.w;
     }
+    __syncthreads();
+    for (int e = threadIdx.x; e < 64 * 16; e += 256) {
+        const int r = e >> 4, c = (e & 15) * 4;
+        const int64_t i = r0 + r, j = c0 + c;
+        if (i >= K || j >= K) continue;
+        float v[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) v[q] = (ti < tj || r <= c + q) ? t[r][c + q] : t[c + q][r];
+        store(i * K + j, v);
+    }
+    if (ti == tj) return;
+    for (int e = threadIdx.x; e < 64 * 16; e += 256) {
+        const int r = e >> 4, c = (e & 15) * 4;
+        const int64_t i = c0 + r, j = r0 + c;     // mirror tile: S(i, j) = S(j, i) = t[j - r0][i - c0]
+        if (i >= K || j >= K) continue;
+        float v[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) v[q] = t[c + q][r];
+        store(i * K + j, v);
+    }
+}
+
+struct StoreF64 {
+    double* C;
+    double scale;
+    __device__ void operator()(int64_t e, const float* v) const
+    {
+        double2* d = reinterpret_cast<double2*>(C + e);
+        d[0] = make_double2(scale * static_cast<double>(v[0]), scale * static_cast<double>(v[1]));
+        d[1] = make_double2(scale * static_cast<double>(v[2]), scale * static_cast<double>(v[3]));
+    }
+};
+
+struct StoreSplitBf16 {
+    __nv_bfloat16* hi;
+    __nv_bfloat16* lo;
+    float scale;
+    __device__ void operator()(int64_t e, const float* v) const
+    {
+        __nv_bfloat16 h[4], l[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float x = scale * v[q];
+            h[q] = __float2bfloat16_rn(x);
+            // x - h is exact in fp32 (h is x rounded to 8 significant bits)
+            l[q] = __float2bfloat16_rn(x - __bfloat162float(h[q]));
+        }
+        *reinterpret_cast<uint2*>(hi + e) = *reinterpret_cast<const uint2*>(h);
+        *reinterpret_cast<uint2*>(lo + e) = *reinterpret_cast<const uint2*>(l);
+    }
+};
+
+static dim3 sym_grid(int64_t K)
+{
+    const unsigned t = static_cast<unsigned>((K + 63) / 64);
+    return dim3(t, t);
 }
 
 cudaError_t launch_sym_full_f64(const float* Su, int64_t K, double scale, double* C, cudaStream_t stream)
 {
     if (K <= 0) return cudaSuccess;
-    const int64_t blocks = std::min<int64_t>((K * K + 255) / 256, 65536);
-    sym_full_f64_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(Su, K, scale, C);
+    if (K % 4 != 0 || (K + 63) / 64 > 65535) return cudaErrorInvalidValue;
+    sym_expand_kernel<<<sym_grid(K), 256, 0, stream>>>(Su, K, StoreF64{C, scale});
     return cudaGetLastError();
-}
-
-__global__ void sym_split_bf16_kernel(const float* __restrict__ Su, int64_t K, float scale,
-                                      __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo)
-{
-    for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < K * K;
-         e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t i = e / K, j = e - i * K;
-        const float v = scale * (i <= j ? Su[i * K + j] : Su[j * K + i]);
-        const __nv_bfloat16 h = __float2bfloat16_rn(v);
-        hi[e] = h;
-        // v - h is exact in fp32 (h is v rounded to 8 significant bits)
-        lo[e] = __float2bfloat16_rn(v - __bfloat162float(h));
-    }
 }
 
 cudaError_t launch_sym_split_bf16(const float* Su, int64_t K, float scale, void* hi, void* lo, cudaStream_t stream)
 {
     if (K <= 0) return cudaSuccess;
-    const int64_t blocks = std::min<int64_t>((K * K + 255) / 256, 65536);
-    sym_split_bf16_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
-        Su, K, scale, static_cast<__nv_bfloat16*>(hi), static_cast<__nv_bfloat16*>(lo));
+    if (K % 4 != 0 || (K + 63) / 64 > 65535) return cudaErrorInvalidValue;
+    sym_expand_kernel<<<sym_grid(K), 256, 0, stream>>>(
+        Su, K, StoreSplitBf16{static_cast<__nv_bfloat16*>(hi), static_cast<__nv_bfloat16*>(lo), scale});
     return cudaGetLastError();
 }
 

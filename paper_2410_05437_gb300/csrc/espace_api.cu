@@ -175,7 +175,7 @@ struct espace_calib_s {
     void* gn = nullptr;            // scratch for normalized gradients (NL-MSE)
     int64_t gn_tokens = 0;
     float* nl_f32 = nullptr;       // NL-MSE scratch: two K x K fp32 autocorrelations
-    void* nl_bf = nullptr;         //   and four K x K bf16 halves (hi / lo of each)
+    void* nl_bf = nullptr;         //   and four bf16 halves (hi / lo of each), Kp x K, zero rows past K
 };
 
 struct espace_proj_s {
@@ -362,11 +362,16 @@ int espace_calib_accumulate_nl(espace_calib_t h, const void* X_dev, const void* 
         X_dev = h->xn;
         G_dev = h->gn;
     }
+    // the bf16 halves of A and B as four blocks of Kp = ceil(K / 64) * 64 rows; the rows past
+    // K stay zero, so that every block is a whole number of 64-row k-blocks
+    const int64_t Kp = (K + 63) / 64 * 64, blk = Kp * K;
     if (h->nl_f32 == nullptr) {
         cudaError_t e = cudaMalloc(&h->nl_f32, sizeof(float) * 2 * kk);
-        if (e == cudaSuccess) e = cudaMalloc(&h->nl_bf, sizeof(uint16_t) * 4 * kk);
+        if (e == cudaSuccess) e = cudaMalloc(&h->nl_bf, sizeof(uint16_t) * 4 * blk);
+        if (e == cudaSuccess) e = cudaMemsetAsync(h->nl_bf, 0, sizeof(uint16_t) * 4 * blk, st);
         if (e != cudaSuccess) {
             if (h->nl_f32) cudaFree(h->nl_f32);
+            if (h->nl_bf) cudaFree(h->nl_bf);
             h->nl_f32 = nullptr;
             h->nl_bf = nullptr;
             return fail(ESPACE_ERR_NOMEM, "espace_calib_accumulate_nl: scratch: %s", cudaGetErrorString(e));
@@ -375,22 +380,22 @@ int espace_calib_accumulate_nl(espace_calib_t h, const void* X_dev, const void* 
     float* a32 = h->nl_f32;
     float* b32 = h->nl_f32 + kk;
     uint16_t* a_hi = static_cast<uint16_t*>(h->nl_bf);
-    uint16_t* a_lo = a_hi + kk;
-    uint16_t* b_hi = a_lo + kk;
-    uint16_t* b_lo = b_hi + kk;
+    uint16_t* a_lo = a_hi + blk;
+    uint16_t* b_hi = a_lo + blk;
+    uint16_t* b_lo = b_hi + blk;
     const int k = static_cast<int>(K);
     // A = X^T X / T and B = G^T G / T (upper triangles on the tensor cores, then the full
     // symmetric matrices split into bf16 hi + lo)
-    CUDA_TRY(launch_zero_f32(h->nl_f32, 2 * kk, st), "accumulate_nl: clear");
-    CUDA_TRY(launch_syrk_upper(X_dev, T, k, a32, st), "accumulate_nl: X^T X");
-    CUDA_TRY(launch_syrk_upper(G_dev, T, k, b32, st), "accumulate_nl: G^T G");
+    CUDA_TRY(launch_syrk_upper_two(X_dev, G_dev, T, k, a32, b32, true, st), "accumulate_nl: X^T X and G^T G");
     CUDA_TRY(launch_sym_split_bf16(a32, K, 1.0f / static_cast<float>(T), a_hi, a_lo, st), "accumulate_nl: split A");
     CUDA_TRY(launch_sym_split_bf16(b32, K, 1.0f / static_cast<float>(T), b_hi, b_lo, st), "accumulate_nl: split B");
     // S += (A B + B A), upper triangle: A B ~ A_hi B_hi + A_hi B_lo + A_lo B_hi and the same
-    // for B A; A and B are symmetric, so S += U^T V with U, V one of them each is S += U V
-    const uint16_t* pairs[6][2] = {{a_hi, b_hi}, {a_hi, b_lo}, {a_lo, b_hi}, {b_hi, a_hi}, {b_hi, a_lo}, {b_lo, a_hi}};
-    for (auto& pr : pairs)
-        CUDA_TRY(launch_syrk_cross_upper(pr[0], pr[1], K, k, h->S, st), "accumulate_nl: product");
+    // for B A; A and B are symmetric, so S += U^T V with U, V one of them each is S += U V,
+    // and the six products are one reduction over six K-row segments of the four blocks
+    const int r = static_cast<int>(Kp);
+    const int seg_u[6] = {0, 0, r, 2 * r, 2 * r, 3 * r};       // A_hi A_hi A_lo B_hi B_hi B_lo
+    const int seg_v[6] = {2 * r, 3 * r, 2 * r, 0, r, 0};       // B_hi B_lo B_hi A_hi A_lo A_hi
+    CUDA_TRY(launch_syrk_segments_upper(h->nl_bf, 4 * Kp, k, r, 6, seg_u, seg_v, h->S, st), "accumulate_nl: products");
     h->mode = mode;
     h->n += 1;
     return ESPACE_OK;

@@ -71,8 +71,18 @@ cudaError_t launch_gemm_nn(const void* A, int64_t lda, const void* B, int64_t ld
 cudaError_t launch_gemm_tn_tokens_f32(const void* U, int R, const void* V, int C, int64_t N, float* out,
                                      int64_t ldo, cudaStream_t stream);
 
+// S's upper triangle += that of sum_q U_q^T V_q, one launch: U_q and V_q are the seg_rows x K
+// blocks of Q ([q_rows][K] bf16, rows contiguous) that start at rows seg_u[q] and seg_v[q]
+// (multiples of 64, as is seg_rows; rows of a block past its data must be zero). At most 6
+// segments.
+cudaError_t launch_syrk_segments_upper(const void* Q, int64_t q_rows, int K, int seg_rows, int nseg,
+                                       const int* seg_u, const int* seg_v, float* S, cudaStream_t stream);
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
+// Two independent SYRKs in one launch: Sx += X^T X and Sy += Y^T Y (upper triangles), or
+// Sx = X^T X and Sy = Y^T Y with assign (the lower triangles are then left unset).
+cudaError_t launch_syrk_upper_two(const void* X, const void* Y, int64_t N, int K, float* Sx, float* Sy,
+                                  bool assign, cudaStream_t stream);
 // The same kernel with two operands: S's upper triangle += that of X^T Y (X, Y [N][K] bf16).
 cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream);
 

@@ -348,6 +348,7 @@ constexpr int SYRK_CHUNK = 16;
 constexpr int PAIR_GROUP_M = 8;
 // Diagonal blocks of a block-diagonal product (one per tensor-parallel rank).
 constexpr int PAIR_MAX_BLOCKS = 8;
+constexpr int PAIR_MAX_SEGS = 6;
 
 template <bool SYRK>
 struct PairShape {
@@ -364,7 +365,9 @@ struct PairProblem {
     const int2* tile_list;   // (tile row, tile col) pairs, or nullptr for the full grid
     void* out;
     int64_t ldo;
-    int upper;               // token-reduction (M/N-major) programs: add only column >= row
+    // token-reduction (M/N-major) programs: bit 0 = add only column >= row; bit 1 (with
+    // ksplit == 1 only) = store the tile instead of adding it
+    int upper;
 };
 
 // A program of one product, or of two where the second one's A operand is the first one's
@@ -393,7 +396,32 @@ struct PairArgs {
     int ak0[PAIR_MAX_BLOCKS];
     int c0[PAIR_MAX_BLOCKS];
     int cw[PAIR_MAX_BLOCKS];
+    // token-reduction programs: when seg_kb > 0, k-block kb reads A's token rows from
+    // seg_a[kb / seg_kb] and B's from seg_b[kb / seg_kb], plus (kb % seg_kb) * BK
+    int seg_kb;
+    int seg_a[PAIR_MAX_SEGS];
+    int seg_b[PAIR_MAX_SEGS];
 };
+
+// First token row of k-block kb in A's and in B's map (segmented token reductions).
+__device__ __forceinline__ void pair_seg_rows(const PairArgs& a, int kb, int& ya, int& yb)
+{
+    if (a.seg_kb <= 0) {
+        ya = yb = kb * BK;
+        return;
+    }
+    const int seg = kb / a.seg_kb;
+    const int off = (kb - seg * a.seg_kb) * BK;
+    int sa = 0, sb = 0;
+#pragma unroll
+    for (int q = 0; q < PAIR_MAX_SEGS; ++q)
+        if (q == seg) {
+            sa = a.seg_a[q];
+            sb = a.seg_b[q];
+        }
+    ya = sa + off;
+    yb = sb + off;
+}
 
 // Column tile tn of problem prob -> A's k offset, B's first row, the first output column
 // and the end of the output columns that tile may store. Unrolled selects keep the block
@@ -456,7 +484,10 @@ __device__ __forceinline__ void pair_decode(const PairArgs& a, int item, int& pr
     prob = item < n0 ? 0 : 1;
     const PairProblem p = pair_problem_of(a, prob);
     const int j = prob == 0 ? item : item - n0;
-    const int tile = j / p.ksplit, split = j - tile * p.ksplit;
+    // split-major: consecutive items are consecutive tiles over the same token range, so a
+    // wave shares that operand slab in L2 and the splits of one tile, which add into the
+    // same output, run at different times
+    const int split = j / p.num_tiles, tile = j - split * p.num_tiles;
     if (p.tile_list != nullptr) {
         const int2 t = p.tile_list[tile];
         tm = t.x;
@@ -570,7 +601,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                 pair_decode(args, item, prob, tm, tn, kb0, kb1);
                 const CUtensorMap* ma = prob == 0 ? &map_a0 : &map_a1;
                 const CUtensorMap* mb = prob == 0 ? &map_b0 : &map_b1;
-                if (prob == 1) {
+                if (prob == 1 && args.ready != nullptr) {
                     // row block tm of A (= product 0's output) must be complete: every
                     // epilogue warp of both CTAs of every tile in it has signalled
                     const int target = 2 * (EPI_THREADS / 32) * args.p[0].tiles_n;
@@ -606,16 +637,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                     uint8_t* sb = sa + PAIR_A_BYTES;
                     if (leader) mbar_arrive_expect_tx(&full[stage], 2 * PAIR_STAGE_BYTES);
                     const uint32_t bar = mapa_shared(smem_u32(&full[stage]), 0);
+                    int ya = kb * BK, yb = kb * BK;
+                    if (SYRK) pair_seg_rows(args, kb, ya, yb);
                     if (SYRK) {
                         // 64 features x 64 tokens per box; the second 64 features at +8 KB
-                        tma_load_2d_pair(sa, ma, bar, row_a, kb * BK);
-                        tma_load_2d_pair(sa + 8192, ma, bar, row_a + 64, kb * BK);
+                        tma_load_2d_pair(sa, ma, bar, row_a, ya);
+                        tma_load_2d_pair(sa + 8192, ma, bar, row_a + 64, ya);
                     } else {
                         tma_load_2d_pair(sa, ma, bar, ak0 + kb * BK, row_a);
                     }
                     if (B_MN) {
-                        tma_load_2d_pair(sb, mb, bar, row_b, kb * BK);
-                        tma_load_2d_pair(sb + 8192, mb, bar, row_b + 64, kb * BK);
+                        tma_load_2d_pair(sb, mb, bar, row_b, yb);
+                        tma_load_2d_pair(sb + 8192, mb, bar, row_b + 64, yb);
                     } else {
                         tma_load_2d_pair(sb, mb, bar, kb * BK, row_b);
                     }
@@ -730,23 +763,38 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                 }
             }
             if (!ok) break;
-            // S[row][col] += run (for col >= row only when the problem is a triangle), 16
-            // bytes at a time
+            // S[row][col] += run, or = run for a program that assigns (for col >= row only
+            // when the problem is a triangle), 16 bytes at a time
             const int row = tm * PAIR_BM + row_in_tile;
             if (row < pb.rows) {
                 float* s_row = reinterpret_cast<float*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
                 const int colb = tn * PAIR_BN + half * 128;
-                const int cmin = pb.upper ? row : 0;
+                const int cmin = (pb.upper & 1) ? row : 0;
+                if (pb.upper & 2) {
 #pragma unroll
-                for (int i = 0; i < 128; i += 4) {
-                    const int col = colb + i;
-                    if (col >= cmin && col + 3 < pb.cols) {
-                        atomicAdd(reinterpret_cast<float4*>(s_row + col),
-                                  make_float4(run[i], run[i + 1], run[i + 2], run[i + 3]));
-                    } else {
+                    for (int i = 0; i < 128; i += 4) {
+                        const int col = colb + i;
+                        if (col >= cmin && col + 3 < pb.cols) {
+                            *reinterpret_cast<float4*>(s_row + col) =
+                                make_float4(run[i], run[i + 1], run[i + 2], run[i + 3]);
+                        } else {
 #pragma unroll
-                        for (int j = 0; j < 4; ++j)
-                            if (col + j >= cmin && col + j < pb.cols) atomicAdd(s_row + col + j, run[i + j]);
+                            for (int j = 0; j < 4; ++j)
+                                if (col + j >= cmin && col + j < pb.cols) s_row[col + j] = run[i + j];
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 128; i += 4) {
+                        const int col = colb + i;
+                        if (col >= cmin && col + 3 < pb.cols) {
+                            atomicAdd(reinterpret_cast<float4*>(s_row + col),
+                                      make_float4(run[i], run[i + 1], run[i + 2], run[i + 3]));
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                if (col + j >= cmin && col + j < pb.cols) atomicAdd(s_row + col + j, run[i + j]);
+                        }
                     }
                 }
             }
@@ -804,7 +852,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                 acc = 0;
                 acc_phase ^= 1u;
             }
-            if (prob == 0 && args.nprob > 1) {
+            if (prob == 0 && args.nprob > 1 && args.ready != nullptr) {
                 // publish this warp's 32 rows of the tile to the second product's producers
                 // (per warp, so that no block-wide barrier can wait on a warp that gave up)
                 fence_proxy_async_global();
@@ -1175,15 +1223,28 @@ int2* syrk_tiles(int K, int tile_rows, int tile_cols, int* count)
     return dev;
 }
 
-// Token splits so that there are about two work items per worker, at least 16 k-blocks
-// (1024 tokens) per split.
+// Token splits per tile: the count s that minimises the last worker's time, ceil(tiles s /
+// workers) waves of ceil(kblocks / s) k-blocks plus a per-item epilogue (the atomic adds of
+// a 256 x 256 fp32 tile, taken as 8 k-blocks of MMA), with at least 16 k-blocks (1024
+// tokens) per split; ties go to fewer splits.
 void choose_splits(int kblocks, int tiles, int workers, int* ksplit, int* kb_per_split)
 {
-    const int want = std::max(1, (2 * workers + tiles - 1) / tiles);
-    int kbps = std::max(16, (kblocks + want - 1) / want);
-    kbps = std::min(kbps, kblocks);
-    *kb_per_split = kbps;
-    *ksplit = (kblocks + kbps - 1) / kbps;
+    constexpr int64_t EPILOGUE_KB = 8;
+    int best_s = 1;
+    int64_t best = INT64_MAX;
+    for (int s = 1; s <= 64; ++s) {
+        const int kbps = (kblocks + s - 1) / s;
+        if (s > 1 && kbps < 16) break;
+        if ((kblocks + kbps - 1) / kbps != s) continue;   // the same split as a smaller s
+        const int64_t waves = (static_cast<int64_t>(tiles) * s + workers - 1) / workers;
+        const int64_t cost = waves * (kbps + EPILOGUE_KB);
+        if (cost < best) {
+            best = cost;
+            best_s = s;
+        }
+    }
+    *ksplit = best_s;
+    *kb_per_split = (kblocks + best_s - 1) / best_s;
 }
 
 }  // namespace
@@ -1191,6 +1252,111 @@ void choose_splits(int kblocks, int tiles, int workers, int* ksplit, int* kb_per
 cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream)
 {
     return launch_syrk_cross_upper(X, X, N, K, S, stream);
+}
+
+cudaError_t launch_syrk_upper_two(const void* X, const void* Y, int64_t N, int K, float* Sx, float* Sy,
+                                  bool assign, cudaStream_t stream)
+{
+    if (N <= 0) return cudaSuccess;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    const int kblocks = static_cast<int>((N + BK - 1) / BK);
+    int ksplit = 1, kbps = kblocks;
+    const bool pair = K > 128 && dev->num_sms >= 2 && pair_kernel_enabled();
+    if (pair) {
+        int count = 0;
+        if (syrk_tiles(K, PAIR_BM, PAIR_BN, &count) == nullptr) return cudaErrorMemoryAllocation;
+        choose_splits(kblocks, 2 * count, dev->num_sms / 2, &ksplit, &kbps);
+    }
+    if (assign && (!pair || ksplit > 1)) {
+        // split reductions add: start from zero
+        const int64_t kk = static_cast<int64_t>(K) * K;
+        cudaError_t e = launch_zero_f32(Sx, kk, stream);
+        if (e == cudaSuccess) e = launch_zero_f32(Sy, kk, stream);
+        if (e != cudaSuccess) return e;
+    }
+    if (!pair) {
+        cudaError_t e = launch_syrk_upper(X, N, K, Sx, stream);
+        return e != cudaSuccess ? e : launch_syrk_upper(Y, N, K, Sy, stream);
+    }
+    int count = 0;
+    const int2* tiles = syrk_tiles(K, PAIR_BM, PAIR_BN, &count);
+    if (tiles == nullptr) return cudaErrorMemoryAllocation;
+    CUtensorMap maps[4];
+    if (!encode_map(&maps[0], X, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
+    if (!encode_map(&maps[2], Y, K, static_cast<uint64_t>(N), K, 64, BK)) return cudaErrorInvalidValue;
+    maps[1] = maps[0];
+    maps[3] = maps[2];
+    PairArgs a{};
+    float* outs[2] = {Sx, Sy};
+    for (int q = 0; q < 2; ++q) {
+        PairProblem& p = a.p[q];
+        p.rows = K;
+        p.cols = K;
+        p.kblocks = kblocks;
+        p.tiles_n = 0;
+        p.num_tiles = count;
+        p.ksplit = ksplit;
+        p.kb_per_split = kbps;
+        p.tile_list = tiles;
+        p.out = outs[q];
+        p.ldo = K;
+        p.upper = assign && ksplit == 1 ? 3 : 1;
+    }
+    a.nprob = 2;       // independent problems: no ready counters
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return launch_pair<true>(maps, a, dev, stream);
+}
+
+cudaError_t launch_syrk_segments_upper(const void* Q, int64_t q_rows, int K, int seg_rows, int nseg,
+                                       const int* seg_u, const int* seg_v, float* S, cudaStream_t stream)
+{
+    if (nseg <= 0) return cudaSuccess;
+    if (nseg > PAIR_MAX_SEGS || seg_rows <= 0 || seg_rows % BK != 0 || K <= 0) return cudaErrorInvalidValue;
+    for (int q = 0; q < nseg; ++q)
+        if (seg_u[q] < 0 || seg_v[q] < 0 || seg_u[q] % BK != 0 || seg_v[q] % BK != 0 ||
+            seg_u[q] + seg_rows > q_rows || seg_v[q] + seg_rows > q_rows)
+            return cudaErrorInvalidValue;
+    DeviceInfo* dev = nullptr;
+    if (device_info(&dev) != ESPACE_OK) return cudaErrorUnknown;
+    if (K <= 128 || dev->num_sms < 2 || !pair_kernel_enabled()) {
+        // one two-operand SYRK per segment
+        const size_t ld = static_cast<size_t>(K);
+        for (int q = 0; q < nseg; ++q) {
+            const auto* base = static_cast<const uint16_t*>(Q);
+            cudaError_t e = launch_syrk_cross_upper(base + seg_u[q] * ld, base + seg_v[q] * ld, seg_rows, K, S, stream);
+            if (e != cudaSuccess) return e;
+        }
+        return cudaSuccess;
+    }
+    int count = 0;
+    const int2* tiles = syrk_tiles(K, PAIR_BM, PAIR_BN, &count);
+    if (tiles == nullptr) return cudaErrorMemoryAllocation;
+    CUtensorMap maps[4];
+    if (!encode_map(&maps[0], Q, K, static_cast<uint64_t>(q_rows), K, 64, BK)) return cudaErrorInvalidValue;
+    maps[1] = maps[2] = maps[3] = maps[0];
+    PairArgs a{};
+    PairProblem& p = a.p[0];
+    p.rows = K;
+    p.cols = K;
+    p.kblocks = nseg * (seg_rows / BK);
+    p.tiles_n = 0;
+    p.num_tiles = count;
+    choose_splits(p.kblocks, count, dev->num_sms / 2, &p.ksplit, &p.kb_per_split);
+    p.tile_list = tiles;
+    p.out = S;
+    p.ldo = K;
+    p.upper = 1;
+    a.nprob = 1;
+    a.seg_kb = seg_rows / BK;
+    for (int q = 0; q < nseg; ++q) {
+        a.seg_a[q] = seg_u[q];
+        a.seg_b[q] = seg_v[q];
+    }
+    a.status = dev->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return launch_pair<true>(maps, a, dev, stream);
 }
 
 cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream)

@@ -416,6 +416,26 @@ def _unit_rows_bf16(A):
     return oracle.bf16_round(np.where(n > 0, A / np.where(n > 0, n, 1.0), 0.0))
 
 
+def test_calib_nl_mse_split_reduction(esp):
+    """NL-MSE terms whose SYRKs split their token reduction (2048 tokens, 15 upper tiles of
+    a ragged K = 1040 per problem, both problems in one launch) and whose K x K products
+    end in a ragged k-block, against the oracle."""
+    K, T = 1040, 2048
+    Xs = synth.ActivationModel(K, seed=71).sample(T, stream="calib_tokens")
+    Gs = (synth.ActivationModel(K, seed=72, outliers=0, lognormal_sigma=0.0)
+          .sample(T, stream="calib_tokens", chunk=1) * 0.01).to(torch.bfloat16)
+    h = esp.espace_calib_create(K)
+    try:
+        esp.espace_calib_accumulate_nl(h, dev(Xs), dev(Gs))
+        C, n = esp.espace_calib_read(h, K)
+        assert n == 1
+    finally:
+        esp.espace_calib_destroy(h)
+    C_o = oracle.nl_mse_term(f64(Xs), f64(Gs))
+    err = np.linalg.norm(C - C_o) / np.linalg.norm(C_o)
+    assert err <= 1e-4, err
+
+
 @pytest.mark.parametrize("normalized", [False, True])
 def test_calib_nl_mse_matches_oracle(esp, normalized):
     """Three calibration sequences of activations and synthetic loss gradients: C (the mean
