@@ -42,7 +42,7 @@ SETS = 4
 
 # DRAM bytes (read + write) of one launch of the dominant kernel at this workload, from the
 # ncu capture summarized in profiles/fused_forward_llama2_qkv_prefill.md (same kernel build).
-FUSED_FORWARD_TRAFFIC_BYTES = 156720384 + 77044480
+FUSED_FORWARD_TRAFFIC_BYTES = 156578560 + 76974848
 
 
 def parse():

@@ -396,9 +396,11 @@ struct PairArgs {
     int ak0[PAIR_MAX_BLOCKS];
     int c0[PAIR_MAX_BLOCKS];
     int cw[PAIR_MAX_BLOCKS];
-    // token-reduction programs: when seg_kb > 0, k-block kb reads A's token rows from
-    // seg_a[kb / seg_kb] and B's from seg_b[kb / seg_kb], plus (kb % seg_kb) * BK
-    int seg_kb;
+    // token-reduction programs: when seg_n > 0, k-block kb is 64-row slab kb / seg_n of
+    // segment kb % seg_n, whose A rows start at seg_a[kb % seg_n] and B rows at seg_b[..]:
+    // the segments' products over one slab run back to back, so that the operand slabs they
+    // share are read from L2
+    int seg_n;
     int seg_a[PAIR_MAX_SEGS];
     int seg_b[PAIR_MAX_SEGS];
 };
@@ -406,12 +408,13 @@ struct PairArgs {
 // First token row of k-block kb in A's and in B's map (segmented token reductions).
 __device__ __forceinline__ void pair_seg_rows(const PairArgs& a, int kb, int& ya, int& yb)
 {
-    if (a.seg_kb <= 0) {
+    if (a.seg_n <= 0) {
         ya = yb = kb * BK;
         return;
     }
-    const int seg = kb / a.seg_kb;
-    const int off = (kb - seg * a.seg_kb) * BK;
+    const int slab = kb / a.seg_n;
+    const int seg = kb - slab * a.seg_n;
+    const int off = slab * BK;
     int sa = 0, sb = 0;
 #pragma unroll
     for (int q = 0; q < PAIR_MAX_SEGS; ++q)
@@ -1226,7 +1229,7 @@ int2* syrk_tiles(int K, int tile_rows, int tile_cols, int* count)
 // Token splits per tile: the count s that minimises the last worker's time, ceil(tiles s /
 // workers) waves of ceil(kblocks / s) k-blocks plus a per-item epilogue (the atomic adds of
 // a 256 x 256 fp32 tile, taken as 8 k-blocks of MMA), with at least 16 k-blocks (1024
-// tokens) per split; ties go to fewer splits.
+// tokens) per split; more splits are taken only for a modelled gain of 2% or more.
 void choose_splits(int kblocks, int tiles, int workers, int* ksplit, int* kb_per_split)
 {
     constexpr int64_t EPILOGUE_KB = 8;
@@ -1238,7 +1241,7 @@ void choose_splits(int kblocks, int tiles, int workers, int* ksplit, int* kb_per
         if ((kblocks + kbps - 1) / kbps != s) continue;   // the same split as a smaller s
         const int64_t waves = (static_cast<int64_t>(tiles) * s + workers - 1) / workers;
         const int64_t cost = waves * (kbps + EPILOGUE_KB);
-        if (cost < best) {
+        if (cost * 50 < best * 49) {
             best = cost;
             best_s = s;
         }
@@ -1349,7 +1352,7 @@ cudaError_t launch_syrk_segments_upper(const void* Q, int64_t q_rows, int K, int
     p.ldo = K;
     p.upper = 1;
     a.nprob = 1;
-    a.seg_kb = seg_rows / BK;
+    a.seg_n = nseg;
     for (int q = 0; q < nseg; ++q) {
         a.seg_a[q] = seg_u[q];
         a.seg_b[q] = seg_v[q];
