@@ -87,7 +87,8 @@ int espace_calib_accumulate_normalized(espace_calib_t h, const void* X_dev, int6
  * cores (fp32), each split into bf16 hi + lo halves, and the products accumulated as
  * A_hi B_hi + A_hi B_lo + A_lo B_hi (and the same for B A) in fp32: about 2^-16 relative.
  * Cannot be mixed with the other accumulations on one handle (ESPACE_ERR_STATE). The first
- * call allocates 16 K^2 bytes of scratch on the handle (4 T K bytes more when normalized).
+ * call allocates 8 K (K + Kp) bytes of scratch on the handle, Kp = K rounded up to a
+ * multiple of 64 (4 T K bytes more when normalized). Four launches per call.
  * C may be indefinite: espace_build_projection then orders eigenvalues by magnitude. */
 int espace_calib_accumulate_nl(espace_calib_t h, const void* X_dev, const void* G_dev, int64_t T,
                                int normalized, void* stream);

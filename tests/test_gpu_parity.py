@@ -416,11 +416,12 @@ def _unit_rows_bf16(A):
     return oracle.bf16_round(np.where(n > 0, A / np.where(n > 0, n, 1.0), 0.0))
 
 
-def test_calib_nl_mse_split_reduction(esp):
-    """NL-MSE terms whose SYRKs split their token reduction (2048 tokens, 15 upper tiles of
-    a ragged K = 1040 per problem, both problems in one launch) and whose K x K products
-    end in a ragged k-block, against the oracle."""
-    K, T = 1040, 2048
+@pytest.mark.parametrize("K,T", [(1040, 2048), (64, 300)])
+def test_calib_nl_mse_split_reduction(esp, K, T):
+    """NL-MSE terms against the oracle: at K = 1040 the SYRKs split their token reduction
+    (2048 tokens, 15 upper tiles of a ragged K per problem, both problems in one launch) and
+    the K x K products end in a ragged k-block padded with zero rows; at K = 64 the 1-CTA
+    kernels run each product as its own launch."""
     Xs = synth.ActivationModel(K, seed=71).sample(T, stream="calib_tokens")
     Gs = (synth.ActivationModel(K, seed=72, outliers=0, lognormal_sigma=0.0)
           .sample(T, stream="calib_tokens", chunk=1) * 0.01).to(torch.bfloat16)
