@@ -218,6 +218,40 @@ def test_projection_columns_orthonormal_and_signs_normalized():
     assert np.array_equal(P_b, oracle.bf16_round(P))
 
 
+def test_normalize_signs_rules():
+    """Eigenvectors are fixed only up to sign: every output column is its input column or
+    its negation, with the entry of largest magnitude positive and, on a tie of magnitudes,
+    the lowest such index deciding; flipping input columns changes nothing and a second
+    pass is the identity."""
+    r = np.random.default_rng(12)
+    P = r.standard_normal((7, 5))
+    P[:, 3] = [0.5, -0.5, 0.1, 0.2, -0.3, 0.0, 0.25]       # tie: index 0 decides, kept
+    P[:, 4] = [-0.5, 0.5, 0.1, 0.2, -0.3, 0.0, 0.25]       # tie: index 0 decides, flipped
+    Q = oracle.normalize_signs(P)
+    for j in range(5):
+        assert np.array_equal(Q[:, j], P[:, j]) or np.array_equal(Q[:, j], -P[:, j])
+        m = np.max(np.abs(Q[:, j]))
+        i = int(np.flatnonzero(np.abs(Q[:, j]) == m)[0])
+        assert Q[i, j] > 0
+    assert np.array_equal(Q[:, 3], P[:, 3])
+    assert np.array_equal(Q[:, 4], -P[:, 4])
+    flips = np.array([1.0, -1.0, -1.0, 1.0, -1.0])
+    assert np.array_equal(oracle.normalize_signs(P * flips), Q)
+    assert np.array_equal(oracle.normalize_signs(Q), Q)
+
+
+def test_weight_autocorr_brute_force_and_orthogonal_rows():
+    """C_W = W^T W / M (Thm. 2): plain loops over the M weight vectors on a tiny W, and the
+    closed form sqrt(M) Q with orthonormal columns, whose C_W is the identity."""
+    r = np.random.default_rng(13)
+    M, K = 5, 3
+    W = r.standard_normal((M, K))
+    E = [[sum(W[m][i] * W[m][j] for m in range(M)) / M for j in range(K)] for i in range(K)]
+    assert np.allclose(oracle.weight_autocorr(W), np.array(E), rtol=0, atol=1e-14)
+    Q, _ = np.linalg.qr(r.standard_normal((40, 6)))
+    assert np.allclose(oracle.weight_autocorr(math.sqrt(40) * Q), np.eye(6), rtol=0, atol=1e-12)
+
+
 def test_prop1_bounds_hold_per_sample():
     X = _calib(K=20, n=500, seed=10)
     P, _, _, _ = oracle.build_projection(oracle.autocorr_sum(X), X.shape[0], 7)
