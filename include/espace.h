@@ -21,6 +21,9 @@
  *     marked "async" only enqueue work on it; the caller synchronizes before reading results.
  *   - The caller owns X, W, Y and streams. The library owns handles and the device memory
  *     behind them (S, P^T, W'^T, the Z scratch) and frees it in the *_destroy calls.
+ *   - A handle's scratch and sums are shared by its calls: calls on one handle must be
+ *     ordered on the GPU (one stream, or streams that wait on each other) and must not be
+ *     made from two host threads at once; calls on different handles may overlap.
  *   - Every int-returning call returns ESPACE_OK (0) or one of the ESPACE_ERR_* codes below;
  *     nothing throws across the ABI, a rejected argument never launches a kernel, and
  *     espace_last_error() describes the most recent failure of the calling thread.

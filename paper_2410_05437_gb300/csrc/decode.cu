@@ -44,6 +44,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "../../include/espace.h"
@@ -585,9 +586,9 @@ template <int MT, bool HI>
 cudaError_t launch_t(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev, cudaStream_t stream)
 {
     auto kern = decode_kernel<MT, HI>;
-    static bool configured[64] = {};
+    static std::atomic<bool> configured[64];   // per device; a repeated set is harmless
     if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
-    if (!configured[dev->device]) {
+    if (!configured[dev->device].load(std::memory_order_acquire)) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              DEC_SMEM_LIMIT - 1024);
         if (e != cudaSuccess) return e;
@@ -595,7 +596,7 @@ cudaError_t launch_t(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev,
         e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, DEC_THREADS, DEC_SMEM_LIMIT - 1024);
         if (e != cudaSuccess) return e;
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
-        configured[dev->device] = true;
+        configured[dev->device].store(true, std::memory_order_release);
     }
     a.stages = pl.stages;
     a.acc_rows = pl.acc_rows;

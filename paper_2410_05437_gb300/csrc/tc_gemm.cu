@@ -23,6 +23,7 @@
 #include <stdlib.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 #include <vector>
 
@@ -923,15 +924,15 @@ cudaError_t launch_kernel(const CUtensorMap& ma, const CUtensorMap& mb, const Tc
     using Cfg = TcCfg<BN, STAGES>;
     auto kern = tc_gemm_kernel<BN, STAGES, MN_MAJOR, EPI>;
     // per instantiation and device; a race only repeats the idempotent call
-    static bool attr_set[64] = {};
+    static std::atomic<bool> attr_set[64];   // per device; a repeated set is harmless
     int device = 0;
     cudaGetDevice(&device);
     if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
-    if (!attr_set[device]) {
+    if (!attr_set[device].load(std::memory_order_acquire)) {
         cudaError_t e =
             cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM_BYTES);
         if (e != cudaSuccess) return e;
-        attr_set[device] = true;
+        attr_set[device].store(true, std::memory_order_release);
     }
     kern<<<grid, GEMM_THREADS, Cfg::SMEM_BYTES, stream>>>(ma, mb, args);
     return cudaGetLastError();
@@ -959,12 +960,12 @@ cudaError_t launch_pair(const CUtensorMap* maps, PairArgs& a, const DeviceInfo* 
     const int items = a.p[0].num_tiles * a.p[0].ksplit + (a.nprob > 1 ? a.p[1].num_tiles * a.p[1].ksplit : 0);
     const int pairs = std::min(items, dev->num_sms / 2);
     auto kern = tc_gemm_pair_kernel<SYRK, B_MN>;
-    static bool attr_set[64] = {};
+    static std::atomic<bool> attr_set[64];   // per device; a repeated set is harmless
     if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
-    if (!attr_set[dev->device]) {
+    if (!attr_set[dev->device].load(std::memory_order_acquire)) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, PAIR_SMEM_BYTES);
         if (e != cudaSuccess) return e;
-        attr_set[dev->device] = true;
+        attr_set[dev->device].store(true, std::memory_order_release);
     }
     kern<<<2 * pairs, PairShape<SYRK>::THREADS, PAIR_SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
     return cudaGetLastError();
