@@ -267,12 +267,15 @@ int espace_proj_tp_info(espace_proj_t p, int* kind, int* tp);
 /* Async. Y = (P^T W)^T (P^T X) for the N tokens of X_dev ([N][K] bf16) into Y_dev
  * ([N][M] bf16): Z = X P is accumulated in fp32 and rounded to bf16 (the paper computes in
  * BF16, Sec. B.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 16 runs
- * a bandwidth-bound kernel that streams P and W' once; N <= 256 runs two tcgen05 launches
- * with the weights as the 128-row operand (phase 1 splits its reduction over the SMs and
- * adds the fp32 partials in a fixed order, so results are reproducible bit for bit);
- * larger N runs one persistent tcgen05 launch holding both products. N = 0 is a no-op.
- * The first call with a larger N than any before on this handle allocates the Z scratch
- * and, for N <= 256, the split workspace (synchronously); later calls allocate nothing. */
+ * a bandwidth-bound kernel that streams P and W' once (when the layer fits it); N <= 256
+ * runs one tcgen05 launch per product with the weights as the 128-row operand, a product
+ * whose tiles would leave more than half of the SMs idle splitting its reduction over them
+ * (one more launch adds the fp32 partials in a fixed order, so results are reproducible bit
+ * for bit); larger N runs one persistent tcgen05 launch holding both products, except that
+ * a layer with K >= 2 M whose Z has fewer 256 x 256 tiles than a quarter of the SMs runs
+ * phase 1 as a split product and phase 2 on CTA pairs. N = 0 is a no-op. The first call
+ * with a larger N than any before on this handle allocates the Z scratch and the split
+ * workspace (synchronously, so outside a stream capture); later calls allocate nothing. */
 int espace_linear_forward(espace_proj_t p, const void* X_dev, int64_t N, void* Y_dev,
                           void* stream);
 
@@ -335,8 +338,8 @@ int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev, int64_t N,
  * families as the projected layer (N <= 8: the streaming kernel; N <= 256: tcgen05 with
  * the weights as the 128-row operand, the reduction split over the SMs in the same cases
  * as the projected layer's products, with fp32 partials in a per-device workspace that
- * the first such call allocates; above: tcgen05): the baseline the projected layer is
- * measured against. Calls that split share the device's workspace: order them on the GPU
+ * the first such call allocates, or grows, and so must make outside a stream capture;
+ * above: tcgen05): the baseline the projected layer is measured against. Calls that split share the device's workspace: order them on the GPU
  * (one stream, or streams that wait on each other). */
 int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev,
                          int64_t M, void* Y_dev, void* stream);
