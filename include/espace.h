@@ -63,7 +63,8 @@ const char* espace_last_error(void);
  * Calibration (Sec. 3.1, Eq. 4): C = X X^T / n summed over calibration tokens. The paper
  * averages per-batch means; the library keeps the running sum S and the token count n and
  * forms C = S / n, which is the same estimate for equal-size batches and the token-weighted
- * mean otherwise. No mean is subtracted (Sec. 3.2 omits input normalization).
+ * mean otherwise. No mean is subtracted: C is Sec. 3.1's autocorrelation E[x x^T], not a
+ * covariance.
  * ------------------------------------------------------------------------------------- */
 
 /* Creates an accumulator for K-dimensional activations with S = 0, n = 0. Allocates an
