@@ -54,6 +54,54 @@ def test_error_codes_without_gpu():
     assert out.value is None
 
 
+def test_null_handles_and_pointers_are_refused_without_gpu():
+    """Every entry point that takes a handle refuses a null one with ESPACE_ERR_ARG, and the
+    dense entry points refuse null pointers and bad shapes, before any CUDA call."""
+    import paper_2410_05437_gb300 as esp
+    L = esp.lib
+    x = ctypes.c_void_p(256)          # never dereferenced: the calls fail on their first check
+    out = ctypes.c_void_p()
+    i = ctypes.c_int()
+    i64 = ctypes.c_int64()
+    calls = {
+        "espace_calib_accumulate": lambda: L.espace_calib_accumulate(None, x, 8, None),
+        "espace_calib_accumulate_normalized": lambda: L.espace_calib_accumulate_normalized(None, x, 8, None),
+        "espace_calib_accumulate_nl": lambda: L.espace_calib_accumulate_nl(None, x, x, 8, 0, None),
+        "espace_calib_read": lambda: L.espace_calib_read(None, None, None, None),
+        "espace_calib_export": lambda: L.espace_calib_export(None, None, None, None),
+        "espace_calib_import": lambda: L.espace_calib_import(None, None, 0, None),
+        "espace_calib_reset": lambda: L.espace_calib_reset(None, None),
+        "espace_build_projection": lambda: L.espace_build_projection(None, x, 64, 8, None, ctypes.byref(out)),
+        "espace_build_projection_go": lambda: L.espace_build_projection_go(None, x, 64, 8, None, ctypes.byref(out)),
+        "espace_build_projection_tp": lambda: L.espace_build_projection_tp(None, x, 64, 64, esp.TP_ROW, 2, None,
+                                                                          ctypes.byref(out)),
+        "espace_proj_tp_info": lambda: L.espace_proj_tp_info(None, ctypes.byref(i), ctypes.byref(i)),
+        "espace_proj_shape": lambda: L.espace_proj_shape(None, ctypes.byref(i64), ctypes.byref(i64), ctypes.byref(i64)),
+        "espace_proj_eigenvalues": lambda: L.espace_proj_eigenvalues(None, None),
+        "espace_proj_read_P": lambda: L.espace_proj_read_P(None, None),
+        "espace_proj_read_Wfold": lambda: L.espace_proj_read_Wfold(None, None),
+        "espace_proj_export": lambda: L.espace_proj_export(None, None, None, None),
+        "espace_linear_forward": lambda: L.espace_linear_forward(None, x, 8, x, None),
+        "espace_linear_forward_path": lambda: L.espace_linear_forward_path(None, x, 8, x, None, 0),
+        "espace_linear_forward_noalloc": lambda: L.espace_linear_forward_noalloc(None, x, 8, x, None),
+        "espace_linear_forward_host": lambda: L.espace_linear_forward_host(None, x, 8, x, None),
+        "espace_proj_refold": lambda: L.espace_proj_refold(None, x, None),
+        "espace_train_forward": lambda: L.espace_train_forward(None, x, 8, x, x, None),
+        "espace_train_backward": lambda: L.espace_train_backward(None, x, x, 8, x, None),
+        "espace_train_weight_grad": lambda: L.espace_train_weight_grad(None, x, None),
+        "espace_dense_forward": lambda: L.espace_dense_forward(None, 8, 64, x, 64, x, None),
+        "espace_dense_backward": lambda: L.espace_dense_backward(None, 8, x, 64, x, 64, x, x, 0, None),
+    }
+    codes = {name: call() for name, call in calls.items()}
+    assert all(c == 1 for c in codes.values()), codes
+    assert out.value is None
+    assert L.espace_linear_forward_launches(None, 8, 0) == -1
+    assert L.espace_dense_forward(x, -1, 64, x, 64, x, None) == 2          # N < 0
+    assert L.espace_dense_forward(x, 8, 12, x, 64, x, None) == 2           # K not a multiple of 8
+    odd = ctypes.c_void_p(264)                                              # 8-byte aligned only
+    assert L.espace_dense_forward(odd, 8, 64, x, 64, x, None) == 3          # ESPACE_ERR_ALIGN
+
+
 @pytest.mark.parametrize("K", [1, 2, 9, 64, 200])
 def test_host_eigh_matches_oracle_jacobi(K):
     import paper_2410_05437_gb300 as esp
