@@ -1159,7 +1159,18 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
             if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p->s_out, cudaStreamNonBlocking);
             for (cudaEvent_t& ev : p->ev)
                 if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
-            if (e != cudaSuccess) return fail_cuda(e, "espace_linear_forward_host: streams");
+            if (e != cudaSuccess) {
+                // release what was made, so that the next call starts over
+                for (cudaEvent_t& ev : p->ev)
+                    if (ev) {
+                        cudaEventDestroy(ev);
+                        ev = nullptr;
+                    }
+                if (p->s_out) cudaStreamDestroy(p->s_out);
+                if (p->s_in) cudaStreamDestroy(p->s_in);
+                p->s_in = p->s_out = nullptr;
+                return fail_cuda(e, "espace_linear_forward_host: streams");
+            }
         }
         if (p->h_cap < N) {
             CUDA_TRY(cudaStreamSynchronize(st), "espace_linear_forward_host: sync before staging growth");
