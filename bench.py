@@ -317,6 +317,7 @@ def run_ours(args, world, rank, local):
         "roofline": {"kernel": k_name, "bound": "tensor",
                      "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
                      "frac": achieved / peak_tc, "peak_kind": f"{peak_kind} bf16 burst",
+                     "peak_sustained": peak_tc_sus, "frac_of_sustained": achieved / peak_tc_sus,
                      "flops_per_launch": k_flops, "ms_per_launch": k_ms,
                      "traffic": FUSED_FORWARD_TRAFFIC_BYTES if fused else None,
                      "algorithmic_bytes": 2.0 * (N * K + K * L + L * M + N * M)},
