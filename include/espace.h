@@ -340,8 +340,9 @@ int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev, int64_t N,
  * the weights as the 128-row operand, the reduction split over the SMs in the same cases
  * as the projected layer's products, with fp32 partials in a per-device workspace that
  * the first such call allocates, or grows, and so must make outside a stream capture;
- * above: tcgen05): the baseline the projected layer is measured against. Calls that split share the device's workspace: order them on the GPU
- * (one stream, or streams that wait on each other). */
+ * above: tcgen05): the baseline the projected layer is measured against. Calls that split
+ * share the device's workspace: order them on the GPU (one stream, or streams that wait on
+ * each other). */
 int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_dev,
                          int64_t M, void* Y_dev, void* stream);
 
