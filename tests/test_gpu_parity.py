@@ -835,6 +835,42 @@ def test_argument_errors_launch_nothing(esp):
         esp.espace_proj_destroy(p)
 
 
+def test_empty_batches_are_no_ops(esp):
+    """Zero tokens (an empty tensor, whose data pointer is null) is accepted by every entry
+    point that takes a batch and changes nothing; the dense backward without accumulation
+    still clears dW."""
+    K, M, L = 128, 64, 32
+    W = dev(synth.weights(M, K, seed=2))
+    p = esp.espace_proj_from_host(synth.random_projection(K, L, seed=2), W)
+    h = esp.espace_calib_create(K)
+    try:
+        bf = dict(dtype=torch.bfloat16, device="cuda")
+        X0, Y0 = torch.empty((0, K), **bf), torch.empty((0, M), **bf)
+        Z0 = torch.empty((0, 64), **bf)
+        esp.espace_linear_forward(p, X0, Y0)
+        esp.espace_linear_forward_host(p, X0.cpu(), Y0.cpu())
+        esp.espace_dense_forward(X0, W, Y0)
+        esp.espace_train_forward(p, X0, Z0, Y0)
+        esp.espace_train_backward(p, Y0, Z0, X0)
+        esp.espace_calib_accumulate(h, X0)
+        S, n = esp.espace_calib_export(h, K)
+        assert n == 0 and not np.any(S)
+        with pytest.raises(esp.EspaceError) as e:
+            esp.espace_calib_read(h, K)                  # C = S / n needs tokens
+        assert e.value.code == 6
+        dW = torch.full((M, K), 7.0, dtype=torch.float32, device="cuda")
+        esp.espace_dense_backward(Y0, X0, W, X0, dW, accumulate=True)
+        torch.cuda.synchronize()
+        assert bool((dW == 7.0).all())
+        esp.espace_dense_backward(Y0, X0, W, X0, dW, accumulate=False)
+        torch.cuda.synchronize()
+        assert not bool(dW.any())
+        esp.espace_check()
+    finally:
+        esp.espace_calib_destroy(h)
+        esp.espace_proj_destroy(p)
+
+
 def test_bounded_wait_reports_timeout_and_context_survives(esp):
     esp.espace_check()
     esp.espace_debug_wait_timeout(2_000_000)          # 2 ms
