@@ -436,7 +436,7 @@ def tp_projection(esp, kind, tp, K, L, W, seed):
 
 def table2_rows(esp, peak_tc):
     """Table 2's per-rank configurations folded onto one GPU, each GEMM of a transformer
-    block timed alone at batch 1 and the model's sequence length (Sec. B.4), dense against
+    block timed alone at batch 1 and the model's sequence length (App. B.4), dense against
     ESPACE. Column-parallel ranks calibrated by Thm. 1 share one projection (they see the
     same inputs), so those layers are the plain projected layer with the rank's L;
     row-parallel ranks each have their own, which makes the first product block-diagonal."""

@@ -152,7 +152,7 @@ int espace_proj_from_host(int64_t K, int64_t M, int64_t L, const double* P_host,
 
 /* Synchronous. Step 4 above for a projection already on the device in bf16: PT_dev is P_b^T
  * as [L][K] row-major bf16 (the L principal directions as rows, e.g. computed by the caller
- * on the GPU, as the paper does, Sec. B.1); it is copied into the handle (the caller keeps
+ * on the GPU, as the paper does, App. B.1); it is copied into the handle (the caller keeps
  * its buffer) and W' = P_b^T W is folded on the device. Both pointers 16-byte aligned. */
 int espace_proj_from_device(int64_t K, int64_t M, int64_t L, const void* PT_dev,
                             const void* W_dev, void* stream, espace_proj_t* out);
@@ -218,7 +218,7 @@ int espace_dense_backward(const void* dY_dev, int64_t N, const void* X_dev, int6
                           void* stream);
 
 /* ---------------------------------------------------------------------------------------
- * Tensor-parallel layers folded onto one GPU (Sec. B.2, Table 2; latency method of Sec. B.4)
+ * Tensor-parallel layers folded onto one GPU (App. B.2, Table 2; latency method of App. B.4)
  *
  * Under tensor parallelism the paper applies ESPACE per rank, each rank r of tp with its
  * own projection P_r of L components. Folded onto one GPU the layer computes, for
@@ -267,7 +267,7 @@ int espace_proj_tp_info(espace_proj_t p, int* kind, int* tp);
 
 /* Async. Y = (P^T W)^T (P^T X) for the N tokens of X_dev ([N][K] bf16) into Y_dev
  * ([N][M] bf16): Z = X P is accumulated in fp32 and rounded to bf16 (the paper computes in
- * BF16, Sec. B.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 16 runs
+ * BF16, App. B.1), then Y = Z W' is accumulated in fp32 and rounded to bf16. N <= 16 runs
  * a bandwidth-bound kernel that streams P and W' once (when the layer fits it); N <= 256
  * runs one tcgen05 launch per product with the weights as the 128-row operand, a product
  * whose tiles would leave more than half of the SMs idle splitting its reduction over them

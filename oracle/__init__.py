@@ -20,7 +20,7 @@ arrays and chains the steps in the order the paper states them:
 * ``go_mse_matrix`` / ``build_projection_go``  Thm. 2: C = C_X C_W + C_W C_X, P its L
   principal eigenvectors (ordered by |eigenvalue|, as the paper does when C is indefinite);
 * ``forward_tp`` / ``build_projection_tp``  ESPACE applied per tensor-parallel rank
-  (Sec. B.2, Table 2), the ranks folded onto one device (Sec. B.4);
+  (App. B.2, Table 2), the ranks folded onto one device (App. B.4);
 * ``train_backward`` / ``dense_backward``  the training view of Sec. 2.2, Y = W^T (P P^T X)
   with P static: gradients with respect to X and W, in the order that keeps Z;
 * ``nl_mse_term`` / ``order_eigenpairs``  Thm. 2's NL-MSE matrix for one calibration
@@ -246,8 +246,8 @@ def build_projection_go(S, n: int, W, L: int):
 
 
 def forward_tp(X, P_blocks, W, kind: str, round_bf16: bool = True) -> np.ndarray:
-    """ESPACE applied per tensor-parallel rank (Sec. B.2, Table 2), the tp ranks' outputs
-    combined on one device (Sec. B.4). ``P_blocks`` is ``[tp, Kr, L]``: rank r's projection.
+    """ESPACE applied per tensor-parallel rank (App. B.2, Table 2), the tp ranks' outputs
+    combined on one device (App. B.4). ``P_blocks`` is ``[tp, Kr, L]``: rank r's projection.
 
     ``kind == "column"`` (QKV, FC1): rank r holds all K inputs and the output rows
     ``W_r = W[r M/tp : (r+1) M/tp]``; its outputs are the layer of Eq. 3 with ``P_r``

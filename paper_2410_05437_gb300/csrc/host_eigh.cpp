@@ -1,6 +1,6 @@
 // host_eigh.cpp -- fp64 symmetric eigen-decomposition on the host for
 // espace_build_projection (Thm. 1 needs the principal eigenvectors of the K x K
-// autocorrelation; the paper runs this step off the hot path, Sec. B.1).
+// autocorrelation; the paper runs this step off the hot path, App. B.1).
 //
 // Method (Golub & Van Loan, "Matrix Computations", Sec. 8.3):
 //   1. Householder tridiagonalization A = Q T Q^T, one reflector per column;

@@ -224,8 +224,8 @@ DECODE_LAYERS = {
 }
 DECODE_TOKENS = (1, 8, 32, 128, 512)
 
-# Per-layer ESPACE configurations of Table 2 (Sec. B.2): per model the tensor-parallel rank
-# count, the sequence length of the GEMM latency measurement (Sec. B.4: batch 1, 2048
+# Per-layer ESPACE configurations of Table 2 (App. B.2): per model the tensor-parallel rank
+# count, the sequence length of the GEMM latency measurement (App. B.4: batch 1, 2048
 # tokens for GPT3, 4096 for Llama2 and Nemotron4), and per layer (name, kind, K, M, L)
 # with K, M the whole layer's input and output widths and L the per-rank rank; QKV and
 # FC1 are column-parallel, the attention projection and FC2 row-parallel. Also Table 1's

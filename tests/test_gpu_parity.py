@@ -491,7 +491,7 @@ def test_calib_nl_mse_matches_oracle(esp, normalized):
         esp.espace_calib_destroy(h)
 
 
-# ------------------------------------------------------------------ tensor-parallel ranks (Sec. B.2)
+# ------------------------------------------------------------------ tensor-parallel ranks (App. B.2)
 
 TP_CASES = [
     # (kind, tp, N, K, M, L)

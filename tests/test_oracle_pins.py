@@ -385,7 +385,7 @@ def test_go_eigenvalues_ordered_by_magnitude():
     assert np.allclose(P @ np.diag(w) @ P.T, C, atol=1e-12 * np.abs(w).max())
 
 
-# ---------------------------------------------------------------- tensor-parallel ranks (Sec. B.2)
+# ---------------------------------------------------------------- tensor-parallel ranks (App. B.2)
 
 def test_tp_row_brute_force():
     """Row-parallel ranks, straight from the definition with pure-Python loops: rank r owns
