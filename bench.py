@@ -1,17 +1,20 @@
-"""Benchmark of the ESPACE projected linear layer on GB300 (one JSON line on rank 0).
+"""Benchmark of the ESPACE projected linear layer on GB300.
 
-Workload (the metric's configuration): the Llama2-7B-shaped fused QKV projection at prefill,
-K = 4096 in-features, M = 12288 out-features, rank L = 2048 (50 % of K), N = 4096 tokens,
-bf16 inputs, fp32 accumulation, with synthetic activations (power-law spectrum i^-0.8,
-1 % outlier channels x20, log-normal channel scales) and W ~ N(0, 1/K).
+Headline workload: the GPT3-22B / Nemotron4-15B-shaped transformer layer at 16,384 tokens,
+the largest single-GPU configuration of the benchmark: QKV (K = 6144 -> M = 18432), FC1
+(6144 -> 24576) and FC2 (24576 -> 6144), each at rank L = K/2, bf16 inputs, fp32
+accumulation, with synthetic activations (power-law spectrum i^-0.8, 1 % outlier channels
+x20, log-normal channel scales), W ~ N(0, 1/K) and a seeded random P folded on the device.
 
-A step is one espace_linear_forward over the N-token batch: the rank-L projection
-Z = bf16(X P) and the folded product Y = Z W' (Eq. 3). Steps rotate over four independent
-(X, P, W') sets, 392 MB in all, so that no step finds its inputs in the 129 MB L2.
-value = algorithmic TFLOP/s, 2 N (K L + L M) per step, over the K timed steps (max over
-ranks). In the same run, and reported beside it in "rows": the dense W^T X baseline on the
-same tensor-core kernel (speedup = dense time / ESPACE time), the calibration accumulate
-(tcgen05 SYRK, Eq. 4) over 65,536 tokens, and the decode-shaped small-N forward at N = 1.
+A step is one espace_linear_forward per layer over the 16,384-token batch (the rank-L
+projection Z = bf16(X P) and the folded product Y = Z W' of Eq. 3, one persistent launch
+each). value = algorithmic TFLOP/s, sum over the three layers of 2 N (K L + L M) per step,
+over the K timed steps (max over ranks). Every layer's X (>= 201 MB) is larger than the
+129 MB L2, so every step reads its inputs from HBM.
+
+Output: the side measurements first, one compact JSON line each ({"row": ...}), then the
+headline as the LAST line (a few hundred bytes): value, roofline of the dominant kernel,
+e2e through host buffers, cpu_baseline, clocks.
 
 --impl reference times the fp64 CPU oracle (the only reference this method has: the paper
 publishes no code) on a bounded sample of the same workload on the host cores.
@@ -35,25 +38,29 @@ import torch  # noqa: E402
 
 import synth  # noqa: E402
 
-CONFIG = "llama2_qkv_prefill"
-METRIC = "ESPACE linear forward TFLOP/s (Llama2-7B QKV prefill, L=K/2)"
+WORKLOAD = "gpt3_22b_layer_prefill"
+LAYERS = ("gpt3_22b_qkv", "gpt3_22b_fc1", "gpt3_22b_fc2")
+METRIC = "ESPACE linear forward TFLOP/s (GPT3-22B layer: QKV+FC1+FC2 at L=K/2, N=16384)"
 UNIT = "TFLOP/s"
 SETS = 4
 
-# DRAM bytes (read + write) of one launch of the dominant kernel at this workload, from the
-# ncu capture summarized in profiles/fused_forward_llama2_qkv_prefill.md (same kernel build).
-FUSED_FORWARD_TRAFFIC_BYTES = 156578560 + 76974848
+# DRAM bytes (read + write) of the dominant kernel per launch at this workload, averaged
+# over the three layers' launches, from one ncu capture of dram__bytes_read.sum and
+# dram__bytes_write.sum (the gpt3_22b_layer profile case); None until captured for the
+# kernel build that runs.
+FUSED_LAYER_TRAFFIC_BYTES = None
+FUSED_LAYER_TRAFFIC_SOURCE = None
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-rows", action="store_true", help="skip the side measurements")
-    ap.add_argument("--profile-case", choices=["fused", "syrk", "decode", "train", "nl"],
-                    help="run a few launches of one kernel on a small fixed case (for ncu) and exit")
+    ap.add_argument("--profile-case", choices=["gpt3_layer", "fused", "syrk", "decode", "train", "nl", "epilogue"],
+                    help="run a few launches of one kernel on a fixed case (for ncu) and exit")
     return ap.parse_args()
 
 
@@ -87,6 +94,22 @@ def load_peaks():
             d = json.load(f)
         return d.get("bf16_tflops", 1900.0), d.get("bf16_tflops_sustained", 1700.0), d.get("hbm_gbs", 6800.0), "measured"
     return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+def emit(obj):
+    """One compact JSON line on stdout."""
+    print(json.dumps(obj, separators=(",", ":")), flush=True)
+
+
+def rounded(obj, digits=4):
+    """Floats rounded to `digits` significant digits (compact output lines)."""
+    if isinstance(obj, float):
+        return float(f"{obj:.{digits}g}")
+    if isinstance(obj, dict):
+        return {k: rounded(v, digits) for k, v in obj.items()}
+    if isinstance(obj, (list, tuple)):
+        return [rounded(v, digits) for v in obj]
+    return obj
 
 
 class ClockSampler:
@@ -141,197 +164,225 @@ def cuda_events(n):
     return [torch.cuda.Event(enable_timing=True) for _ in range(n)]
 
 
+def layer_shapes():
+    out = []
+    for name in LAYERS:
+        c = synth.CONFIGS[name]
+        out.append((name, c["K"], c["M"], c["L"], c["N"]))
+    return out
+
+
+def step_flops():
+    return sum(2.0 * N * (K * L + L * M) for _, K, M, L, N in layer_shapes())
+
+
 # ----------------------------------------------------------------------------- reference arm
+
+def oracle_sample(tokens, seed):
+    """Per layer of the headline workload: `tokens` tokens of X, a random bf16 P and a
+    random bf16 W' of the layer's shapes (the fold is offline, Sec. 2.2, and the values do
+    not change the oracle's time)."""
+    import oracle
+    out = []
+    for name, K, M, L, N in layer_shapes():
+        rng = np.random.default_rng(seed + K + M)
+        X = synth.bf16_to_f64(synth.ActivationModel(K, seed=seed).sample(tokens))
+        Pb = oracle.bf16_round(rng.standard_normal((K, L)) * K ** -0.5)
+        Wf = oracle.bf16_round(rng.standard_normal((L, M)) * L ** -0.5)
+        out.append((X, Pb, Wf))
+    return out
+
+
+def oracle_step(sample):
+    import oracle
+    for X, Pb, Wf in sample:
+        oracle.contract(oracle.project(X, Pb), Wf)
+
+
+def sample_tokens():
+    return max(1, min(16, os.cpu_count() or 1))
+
 
 def run_reference(args, world, rank):
     """fp64 oracle on the host cores, on a bounded sample of the workload."""
-    import oracle
     if rank != 0:
         return
-    cfg = synth.CONFIGS[CONFIG]
-    K, M, L = cfg["K"], cfg["M"], cfg["L"]
-    seed = synth.config_seed(CONFIG)
-    sample_tokens = 8
-    model = synth.ActivationModel(K, seed=seed)
-    X = synth.bf16_to_f64(model.sample(sample_tokens))
-    W = synth.bf16_to_f64(synth.weights(M, K, seed=seed))
-    Pb = oracle.bf16_round(synth.random_projection(K, L, seed=seed))
-    # W' = P^T W is folded offline (Sec. 2.2); it is an input of the timed forward here
-    Wf = oracle.bf16_round(Pb.T @ W.T)
-    flops_per_token = 2.0 * (K * L + L * M)
+    t = sample_tokens()
+    sample = oracle_sample(t, synth.BASE_SEED + 900)
+    flops = step_flops() / synth.CONFIGS[LAYERS[0]]["N"] * t
     times = []
     for i in range(args.warmup + args.steps):
         t0 = time.perf_counter()
-        Z = oracle.project(X, Pb)
-        oracle.contract(Z, Wf)
+        oracle_step(sample)
         dt = time.perf_counter() - t0
         if i >= args.warmup:
             times.append(dt)
     total = sum(times)
-    value = flops_per_token * sample_tokens * len(times) / total / 1e12
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    sample = f"{sample_tokens} tokens of N={cfg['N']} per step (projection + folded product, fold precomputed)"
-    line = {
+    value = flops * len(times) / total / 1e12
+    cores = min(int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1)), t)
+    desc = f"{t} of 16384 tokens per step through each of QKV, FC1, FC2 (projection + folded product; fold offline)"
+    emit({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic",
-        "config": {"workload": "llama2_7b_qkv_prefill", "K": K, "M": M, "L": L, "N": cfg["N"]},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": min(cores, sample_tokens),
-                         "kind": "oracle", "sample": sample},
+        "data": "synthetic", "config": {"workload": WORKLOAD, "layers": "qkv 6144x18432, fc1 6144x24576, fc2 24576x6144",
+                                        "L": "K/2", "N": 16384},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-    }
-    print(json.dumps(line), flush=True)
+    })
 
 
 def cpu_baseline_leg():
-    import oracle
-    cfg = synth.CONFIGS[CONFIG]
-    K, M, L = cfg["K"], cfg["M"], cfg["L"]
-    seed = synth.config_seed(CONFIG)
-    sample_tokens = 8
-    model = synth.ActivationModel(K, seed=seed)
-    X = synth.bf16_to_f64(model.sample(sample_tokens))
-    W = synth.bf16_to_f64(synth.weights(M, K, seed=seed))
-    Pb = oracle.bf16_round(synth.random_projection(K, L, seed=seed))
-    Wf = oracle.bf16_round(Pb.T @ W.T)
+    t = sample_tokens()
+    sample = oracle_sample(t, synth.BASE_SEED + 900)
+    flops = step_flops() / synth.CONFIGS[LAYERS[0]]["N"] * t
+    oracle_step(sample)                     # first touch of the arrays
     t0 = time.perf_counter()
     reps = 0
     while True:
-        oracle.contract(oracle.project(X, Pb), Wf)
+        oracle_step(sample)
         reps += 1
-        if time.perf_counter() - t0 > 10.0 or reps >= 20:
+        if time.perf_counter() - t0 > 10.0 or reps >= 5:
             break
     dt = time.perf_counter() - t0
-    value = 2.0 * (K * L + L * M) * sample_tokens * reps / dt / 1e12
-    cores = min(os.cpu_count() or 1, sample_tokens)
-    return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{sample_tokens} tokens x {reps} repetitions of the fp64 oracle forward "
-                      f"(projection + folded product) at K={K}, L={L}, M={M}"}
+    return {"value": flops * reps / dt / 1e12, "unit": UNIT, "cores": min(os.cpu_count() or 1, t),
+            "kind": "oracle",
+            "sample": f"{t} tokens x {reps} repetitions through QKV, FC1 and FC2 of the fp64 oracle forward"}
 
 
 # ----------------------------------------------------------------------------- our arm
 
+def build_layers(esp, seed):
+    layers = []
+    for name, K, M, L, N in layer_shapes():
+        X = synth.ActivationModel(K, seed=seed).sample_device(N)
+        W = synth.weights_device(M, K, seed=seed)
+        p = device_projection(esp, K, L, W, seed)
+        Lp = (L + 63) // 64 * 64
+        layers.append({"name": name, "K": K, "M": M, "L": L, "N": N, "X": X, "W": W, "p": p,
+                       "Y": torch.empty((N, M), dtype=torch.bfloat16, device="cuda"),
+                       "flops": 2.0 * N * (K * L + L * M), "dense_flops": 2.0 * N * K * M,
+                       "bytes": 2.0 * (N * K + K * Lp + Lp * M + N * M)})
+    torch.cuda.synchronize()
+    return layers
+
+
 def run_ours(args, world, rank, local):
     import paper_2410_05437_gb300 as esp
     torch.cuda.set_device(local)
-    cfg = synth.CONFIGS[CONFIG]
-    K, M, L, N = cfg["K"], cfg["M"], cfg["L"], cfg["N"]
-    seed = synth.config_seed(CONFIG) + 1000 * rank
+    seed = synth.BASE_SEED + 800 + 1000 * rank
     peak_tc, peak_tc_sus, peak_hbm, peak_kind = load_peaks()
-
-    model = synth.ActivationModel(K, seed=seed)
-    sets = []
-    for s in range(SETS):
-        X = model.sample_device(N, chunk=s)
-        W = synth.weights_device(M, K, seed=seed, chunk=s)
-        P = synth.random_projection(K, L, seed=seed + s)
-        p = esp.espace_proj_from_host(P, W)
-        sets.append({"X": X, "W": W, "p": p, "Y": torch.empty((N, M), dtype=torch.bfloat16, device="cuda")})
-    torch.cuda.synchronize()
-
-    flops = 2.0 * N * (K * L + L * M)
-    flops_phase2 = 2.0 * N * L * M
-    dense_flops = 2.0 * N * K * M
+    layers = build_layers(esp, seed)
+    flops = sum(l["flops"] for l in layers)
+    launches = [esp.espace_linear_forward_launches(l["p"], l["N"]) for l in layers]
 
     sampler = ClockSampler(local)
     sampler.start()
-
-    # ---- warm-up
     for i in range(args.warmup):
-        s = sets[i % SETS]
-        esp.espace_linear_forward(s["p"], s["X"], s["Y"])
+        for l in layers:
+            esp.espace_linear_forward(l["p"], l["X"], l["Y"])
     torch.cuda.synchronize()
 
-    # ---- timed region: exactly K steps
-    starts, mids, ends = cuda_events(args.steps), cuda_events(args.steps), cuda_events(args.steps)
-    for e in mids:
-        e.record()                       # materialize the event handles
+    # ---- timed region: exactly K steps; an event before each layer's launch
+    ev = [cuda_events(len(layers) + 1) for _ in range(args.steps)]
+    for row in ev:
+        for e in row:
+            e.record()                       # materialize the event handles
     torch.cuda.synchronize()
     barrier(world)
     torch.cuda.synchronize()
     t_begin, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_begin.record()
     for i in range(args.steps):
-        s = sets[i % SETS]
-        starts[i].record()
-        esp.espace_set_phase_event(mids[i])
-        esp.espace_linear_forward(s["p"], s["X"], s["Y"])
-        ends[i].record()
+        for j, l in enumerate(layers):
+            ev[i][j].record()
+            esp.espace_linear_forward(l["p"], l["X"], l["Y"])
+        ev[i][-1].record()
     t_end.record()
     torch.cuda.synchronize()
     barrier(world)
     total_ms = max_over_ranks(t_begin.elapsed_time(t_end), world)
-    phase1 = [starts[i].elapsed_time(mids[i]) for i in range(args.steps)]
-    phase2 = [mids[i].elapsed_time(ends[i]) for i in range(args.steps)]
-    step_ms = [starts[i].elapsed_time(ends[i]) for i in range(args.steps)]
+    layer_ms = [[ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(args.steps)] for j in range(len(layers))]
+    step_ms = [ev[i][0].elapsed_time(ev[i][-1]) for i in range(args.steps)]
     ms_per_step = total_ms / args.steps
     value = flops * args.steps * world / (total_ms * 1e-3) / 1e12
     esp.espace_check()
+    clocks = sampler.stop()
 
     # ---- end to end through the C ABI with host buffers (pinned), copies inside the timed
     # region: espace_linear_forward_host copies X in, runs the products and copies Y out,
     # overlapping the copies of some token chunks with the products of others
-    Xh = [s["X"].cpu().pin_memory() for s in sets]
-    Yh = torch.empty((N, M), dtype=torch.bfloat16).pin_memory()
-    e2e_steps = max(3, min(args.steps, 20))
-    for i in range(2):
-        esp.espace_linear_forward_host(sets[i % SETS]["p"], Xh[i % SETS], Yh)
+    Xh = [l["X"].cpu().pin_memory() for l in layers]
+    Yh = [torch.empty((l["N"], l["M"]), dtype=torch.bfloat16).pin_memory() for l in layers]
+    e2e_steps = max(3, min(args.steps, 5))
+    for j, l in enumerate(layers):
+        esp.espace_linear_forward_host(l["p"], Xh[j], Yh[j])
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for i in range(e2e_steps):
-        esp.espace_linear_forward_host(sets[i % SETS]["p"], Xh[i % SETS], Yh)
+        for j, l in enumerate(layers):
+            esp.espace_linear_forward_host(l["p"], Xh[j], Yh[j])
     e1.record()
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world) / e2e_steps
-    e2e_value = flops * world / (e2e_ms * 1e-3) / 1e12
+    h2d = sum(2 * l["N"] * l["K"] for l in layers)
+    d2h = sum(2 * l["N"] * l["M"] for l in layers)
+    del Xh, Yh
 
-    rows = {}
+    # ---- the dense layer on the same kernels (speedup), and the side rows
+    dense_ms = []
+    for l in layers:
+        dense_ms.append(events_ms(lambda i, l=l: esp.espace_dense_forward(l["X"], l["W"], l["Y"]), reps=5, warm=2))
+    esp.espace_check()
+    per_layer = {}
+    for j, l in enumerate(layers):
+        k_ms = statistics.mean(layer_ms[j])
+        per_layer[l["name"]] = {"K": l["K"], "M": l["M"], "L": l["L"], "N": l["N"], "launches": launches[j],
+                                "espace_ms": k_ms, "dense_ms": dense_ms[j], "speedup": dense_ms[j] / k_ms,
+                                "espace_tflops": l["flops"] / k_ms / 1e9,
+                                "frac_tensor_peak": l["flops"] / k_ms / 1e9 / peak_tc}
+    if rank == 0:
+        emit({"row": "gpt3_22b_layer_per_layer", **rounded(per_layer)})
     if not args.no_rows:
-        rows = side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, ms_per_step)
-    clocks = sampler.stop()
-    if not args.no_rows and rank == 0:
-        # the other workloads (after the clock sampler: they are not part of the timed step)
-        rows.update(config_rows(esp, peak_tc, peak_hbm))
+        for name, row in side_rows(esp, args, peak_tc, peak_hbm):
+            if rank == 0:
+                emit({"row": name, **rounded(row)})
+    for l in layers:
+        esp.espace_proj_destroy(l["p"])
+    del layers
 
-    fused = esp.espace_linear_forward_launches(sets[0]["p"], N) == 1
-    if fused:
-        # one persistent launch holds both products: it is the dominant (only) kernel
-        k_ms = statistics.mean(phase2)
-        k_flops = flops
-        k_name = "tc_gemm_pair_kernel (fused forward: Z = X P, then Y = Z W')"
-    else:
-        k_ms = statistics.mean(phase2)
-        k_flops = flops_phase2
-        k_name = "tc_gemm_pair_kernel (phase 2: Y = Z W')"
-    achieved = k_flops / (k_ms * 1e-3) / 1e12
+    # ---- roofline of the dominant kernel: the fused forward (tc_gemm_pair_kernel), one
+    # launch per layer; per launch on average = all three launches' flops over their time
+    fused = all(n == 1 for n in launches)
+    kern_ms = sum(statistics.mean(m) for m in layer_ms)
+    achieved = flops / (kern_ms * 1e-3) / 1e12
+    n_l = len(LAYERS)
+    algo_bytes = sum(2.0 * (N * K + K * L + L * M + N * M) for _, K, M, L, N in layer_shapes()) / n_l
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded power-law activations with outlier channels; random-init W; random orthonormal P)",
-        "config": {"workload": "llama2_7b_qkv_prefill", "K": K, "M": M, "L": L, "N": N,
-                   "tokens_per_step_per_gpu": N, "parallelism": f"replicas{world}",
-                   "l2": f"inputs rotate over {SETS} sets of X, P, W' ({SETS * 2 * (N * K + K * L + L * M) / 1e6:.0f} MB > 129 MB L2)"},
-        "roofline": {"kernel": k_name, "bound": "tensor",
-                     "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
+        "data": "synthetic (seeded power-law activations with outlier channels; random-init W; random P)",
+        "config": {"workload": WORKLOAD, "layers": "qkv 6144x18432, fc1 6144x24576, fc2 24576x6144",
+                   "L": "K/2", "N": 16384, "parallelism": f"replicas{world}",
+                   "l2": "no flush: every layer's X (>= 201 MB) and W' exceed the 129 MB L2"},
+        "roofline": {"kernel": "tc_gemm_pair_kernel (fused forward, one launch per layer)" if fused
+                     else "tc_gemm_pair_kernel (forward launches)",
+                     "bound": "tensor", "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
                      "frac": achieved / peak_tc, "peak_kind": f"{peak_kind} bf16 burst",
-                     "peak_sustained": peak_tc_sus, "frac_of_sustained": achieved / peak_tc_sus,
-                     "flops_per_launch": k_flops, "ms_per_launch": k_ms,
-                     "traffic": FUSED_FORWARD_TRAFFIC_BYTES if fused else None,
-                     "algorithmic_bytes": 2.0 * (N * K + K * L + L * M + N * M)},
-        "phases_ms": {"before_event": statistics.mean(phase1), "after_event": statistics.mean(phase2),
-                      "launches_per_step": 1 if fused else 2},
+                     "frac_of_sustained": achieved / peak_tc_sus,
+                     "flops_per_launch": flops / n_l, "ms_per_launch": kern_ms / n_l,
+                     "traffic": FUSED_LAYER_TRAFFIC_BYTES if fused else None,
+                     "traffic_source": FUSED_LAYER_TRAFFIC_SOURCE if fused else None,
+                     "algorithmic_bytes": algo_bytes},
         "step_ms": {"mean": statistics.mean(step_ms), "median": statistics.median(step_ms),
-                    "min": min(step_ms), "max": max(step_ms), "kernel_median": statistics.median(phase2)},
-        "roofline_step": {"frac_of_tensor_peak": (flops / (ms_per_step * 1e-3) / 1e12) / peak_tc,
-                          "roofline_ms": max(flops / (peak_tc * 1e12),
-                                             2.0 * (N * K + K * L + L * M + N * M) / (peak_hbm * 1e9)) * 1e3},
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": N * K * 2,
-                "d2h_bytes_per_step": N * M * 2, "ms_per_step": e2e_ms},
-        "gpu_launches": (1 if fused else 2) * args.steps,
-        "rows": rows,
+                    "min": min(step_ms), "max": max(step_ms)},
+        "speedup_over_dense": sum(dense_ms) / kern_ms,
+        "e2e": {"value": flops * world / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+                "api": "espace_linear_forward_host, pinned host X and Y"},
+        "gpu_launches": sum(launches) * args.steps,
         "clocks": clocks,
     }
     if rank == 0 and world == 1:
@@ -339,66 +390,55 @@ def run_ours(args, world, rank, local):
             line["cpu_baseline"] = cpu_baseline_leg()
         except Exception as ex:   # the baseline must not sink the GPU line
             line["cpu_baseline"] = {"error": repr(ex)}
-    for s in sets:
-        esp.espace_proj_destroy(s["p"])
     if rank == 0:
-        print(json.dumps(line), flush=True)
+        emit(rounded(line, 6))
 
 
-def side_rows(esp, sets, model, K, M, L, N, args, peak_tc, peak_hbm, flops, espace_ms):
-    rows = {}
-    reps = max(10, args.steps)
-    # dense baseline Y = X W^T on the same kernel
-    for i in range(3):
-        s = sets[i % SETS]
-        esp.espace_dense_forward(s["X"], s["W"], s["Y"])
-    torch.cuda.synchronize()
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record()
-    for i in range(reps):
-        s = sets[i % SETS]
-        esp.espace_dense_forward(s["X"], s["W"], s["Y"])
-    b.record()
-    torch.cuda.synchronize()
-    dense_ms = a.elapsed_time(b) / reps
-    dflops = 2.0 * N * K * M
-    # the same forward on two launches (Z through the scratch buffer), for comparison
-    for i in range(3):
-        s = sets[i % SETS]
-        esp.espace_linear_forward_path(s["p"], s["X"], s["Y"], esp.PATH_TENSOR_SPLIT)
-    torch.cuda.synchronize()
-    a.record()
-    for i in range(reps):
-        s = sets[i % SETS]
-        esp.espace_linear_forward_path(s["p"], s["X"], s["Y"], esp.PATH_TENSOR_SPLIT)
-    b.record()
-    torch.cuda.synchronize()
-    split_ms = a.elapsed_time(b) / reps
-    rows["forward_two_launches"] = {"ms": split_ms, "tflops": flops / split_ms / 1e9}
-    rows["dense_forward"] = {"ms": dense_ms, "tflops": dflops / dense_ms / 1e9,
-                             "frac_tensor_peak": dflops / dense_ms / 1e9 / peak_tc,
-                             "speedup_espace_over_dense": dense_ms / espace_ms}
+def side_rows(esp, args, peak_tc, peak_hbm):
+    """(name, row) pairs of the other workloads: the Llama2-7B QKV prefill layer (fused,
+    two launches, dense, decode sweep), its calibration SYRK, and the rest of the benchmark's
+    workloads (config_rows)."""
+    rows = []
+    K, M, L, N = 4096, 12288, 2048, 4096
+    seed = synth.config_seed("llama2_qkv_prefill")
+    model = synth.ActivationModel(K, seed=seed)
+    # four independent (X, P, W') sets rotate so that no call finds its inputs in L2
+    sets = []
+    for s in range(SETS):
+        W = synth.weights_device(M, K, seed=seed, chunk=s)
+        sets.append({"X": model.sample_device(N, chunk=s), "W": W, "p": device_projection(esp, K, L, W, seed + s),
+                     "Y": torch.empty((N, M), dtype=torch.bfloat16, device="cuda")})
+    try:
+        flops, dflops = 2.0 * N * (K * L + L * M), 2.0 * N * K * M
+        reps = max(10, args.steps)
+        f_ms = events_ms(lambda i: esp.espace_linear_forward(sets[i % SETS]["p"], sets[i % SETS]["X"], sets[i % SETS]["Y"]), reps=reps)
+        s_ms = events_ms(lambda i: esp.espace_linear_forward_path(sets[i % SETS]["p"], sets[i % SETS]["X"], sets[i % SETS]["Y"],
+                                                                  esp.PATH_TENSOR_SPLIT), reps=reps)
+        d_ms = events_ms(lambda i: esp.espace_dense_forward(sets[i % SETS]["X"], sets[i % SETS]["W"], sets[i % SETS]["Y"]), reps=reps)
+        esp.espace_check()
+        rows.append(("llama2_qkv_prefill", {"K": K, "M": M, "L": L, "N": N, "fused_ms": f_ms, "two_launch_ms": s_ms,
+                                            "dense_ms": d_ms, "speedup": d_ms / f_ms,
+                                            "fused_frac_tensor_peak": flops / f_ms / 1e9 / peak_tc,
+                                            "dense_frac_tensor_peak": dflops / d_ms / 1e9 / peak_tc}))
+        rows.append(("decode_sweep_llama2_qkv", decode_sweep(esp, K, M, L, 0, peak_hbm, sets=sets)))
+    finally:
+        for s in sets:
+            esp.espace_proj_destroy(s["p"])
+    del sets
     # calibration: S += X^T X over 65,536 tokens (tcgen05 SYRK)
-    n_cal = synth.CONFIGS[CONFIG]["calib_tokens"]
+    n_cal = synth.CONFIGS["llama2_qkv_prefill"]["calib_tokens"]
     Xc = model.sample_device(n_cal, stream="calib_tokens")
     h = esp.espace_calib_create(K)
-    esp.espace_calib_accumulate(h, Xc)
-    esp.espace_calib_reset(h)
-    torch.cuda.synchronize()
-    crep = 3
-    a.record()
-    for _ in range(crep):
-        esp.espace_calib_accumulate(h, Xc)
-    b.record()
-    torch.cuda.synchronize()
-    cal_ms = a.elapsed_time(b) / crep
-    cflops = float(n_cal) * K * (K + 1)
-    rows["calib_accumulate"] = {"tokens": n_cal, "ms": cal_ms, "tflops_symmetric": cflops / cal_ms / 1e9,
-                                "frac_tensor_peak": cflops / cal_ms / 1e9 / peak_tc}
-    esp.espace_calib_destroy(h)
+    try:
+        cal_ms = events_ms(lambda i: esp.espace_calib_accumulate(h, Xc), reps=3, warm=1)
+        esp.espace_check()
+    finally:
+        esp.espace_calib_destroy(h)
     del Xc
-    # decode-shaped forward, N = 1 .. 512 tokens, on the main workload's rotating sets
-    rows["decode_sweep_llama2_qkv"] = decode_sweep(esp, K, M, L, 0, peak_hbm, sets=sets)
+    cflops = float(n_cal) * K * (K + 1)
+    rows.append(("calib_accumulate_k4096", {"tokens": n_cal, "ms": cal_ms, "tflops_symmetric": cflops / cal_ms / 1e9,
+                                            "frac_tensor_peak": cflops / cal_ms / 1e9 / peak_tc}))
+    rows.extend(config_rows(esp, peak_tc, peak_hbm))
     return rows
 
 
@@ -533,24 +573,21 @@ def decode_sweep(esp, K, M, L, seed, peak_hbm, sets=None):
 
 
 def config_rows(esp, peak_tc, peak_hbm):
-    """The other workloads of the benchmark, as side rows: the Llama2-7B MLP over a rank
-    sweep, the GPT3-22B layer at 16,384 tokens, calibration over 1,048,576 tokens at K = 6144
-    and K = 24576, the decode sweep on the other Llama2-7B layers, and the whole Llama2-7B
-    layer at batch 1, sequence 4096."""
-    rows = {}
+    """(name, row) pairs of the other workloads of the benchmark: the Llama2-7B MLP over a
+    rank sweep, calibration over 1,048,576 tokens at K = 6144 and K = 24576, the decode sweep
+    on the other Llama2-7B layers, the whole Llama2-7B layer at batch 1, sequence 4096,
+    Table 2's folded tensor-parallel layers (one row per model), the NL-MSE calibration and
+    the training step."""
+    rows = []
     seed = synth.BASE_SEED + 500
-    sweep = {}
     for name, (K, M) in (("gate_up", (4096, 22016)), ("down", (11008, 4096))):
+        sweep = {}
         for frac in (0.8, 0.7, 0.6, 0.5):
             L = int(round(frac * K))
-            sweep[f"{name}_{int(frac * 100)}pct"] = layer_row(esp, K, M, L, 8192, seed, peak_tc)
-    rows["llama2_mlp_rank_sweep"] = sweep
-    gpt = {}
-    for name in ("gpt3_22b_qkv", "gpt3_22b_fc1", "gpt3_22b_fc2"):
-        cfg = synth.CONFIGS[name]
-        gpt[name] = layer_row(esp, cfg["K"], cfg["M"], cfg["L"], cfg["N"], seed, peak_tc)
-    rows["gpt3_22b_layer"] = gpt
-    cal = {}
+            r = layer_row(esp, K, M, L, 8192, seed, peak_tc)
+            sweep[f"L{int(frac * 100)}pct"] = {k: r[k] for k in ("L", "espace_ms", "dense_ms", "speedup",
+                                                                 "espace_frac_tensor_peak")}
+        rows.append((f"llama2_mlp_{name}_rank_sweep", {"K": K, "M": M, "N": 8192, **sweep}))
     n_total, chunk = 1 << 20, 65536
     for K in (6144, 24576):
         Xc = synth.ActivationModel(K, seed=seed).sample_device(chunk, stream="calib_tokens")
@@ -564,24 +601,26 @@ def config_rows(esp, peak_tc, peak_hbm):
             esp.espace_calib_destroy(h)
         del Xc
         cflops = float(n_total) * K * (K + 1)
-        cal[str(K)] = {"tokens": n_total, "ms": ms, "tflops_symmetric": cflops / ms / 1e9,
-                       "frac_tensor_peak": cflops / ms / 1e9 / peak_tc,
-                       "note": "16 accumulations of one 65,536-token chunk"}
-    rows["calibration_1m_tokens"] = cal
+        rows.append((f"calibration_1m_tokens_k{K}", {"tokens": n_total, "ms": ms, "tflops_symmetric": cflops / ms / 1e9,
+                                                   "frac_tensor_peak": cflops / ms / 1e9 / peak_tc,
+                                                   "note": "16 accumulations of one 65,536-token chunk"}))
     for name in ("o", "gate_up", "down"):
         K, M = synth.DECODE_LAYERS[name]
-        rows[f"decode_sweep_llama2_{name}"] = decode_sweep(esp, K, M, K // 2, seed, peak_hbm)
+        rows.append((f"decode_sweep_llama2_{name}", decode_sweep(esp, K, M, K // 2, seed, peak_hbm)))
     layer = {}
     for name in ("qkv", "o", "gate_up", "down"):
         K, M = synth.DECODE_LAYERS[name]
-        layer[name] = layer_row(esp, K, M, K // 2, 4096, seed, peak_tc)
-    layer["total"] = {"espace_ms": sum(v["espace_ms"] for v in layer.values()),
-                      "dense_ms": sum(v["dense_ms"] for v in layer.values())}
-    layer["total"]["speedup"] = layer["total"]["dense_ms"] / layer["total"]["espace_ms"]
-    rows["llama2_layer_prefill_batch1_seq4096"] = layer
-    rows["table2_tp_folded_gemm_latency"] = table2_rows(esp, peak_tc)
-    rows["nl_mse_calibration"] = nl_mse_row(esp, peak_tc, seed)
-    rows["training_step"] = training_rows(esp, peak_tc, seed)
+        r = layer_row(esp, K, M, K // 2, 4096, seed, peak_tc)
+        layer[name] = {"espace_ms": r["espace_ms"], "dense_ms": r["dense_ms"]}
+    tot_e = sum(v["espace_ms"] for v in layer.values())
+    tot_d = sum(v["dense_ms"] for v in layer.values())
+    layer["total"] = {"espace_ms": tot_e, "dense_ms": tot_d, "speedup": tot_d / tot_e}
+    rows.append(("llama2_layer_prefill_batch1_seq4096", layer))
+    for model, r in table2_rows(esp, peak_tc).items():
+        rows.append((f"table2_tp_folded_{model}", r))
+    rows.append(("nl_mse_calibration", nl_mse_row(esp, peak_tc, seed)))
+    for name, r in training_rows(esp, peak_tc, seed).items():
+        rows.append((f"training_step_{name}", r))
     return rows
 
 
@@ -682,12 +721,29 @@ def graph_time_us(call, per_graph=20, replays=10):
 
 def profile_case(which):
     """A few launches of one kernel, with little else on the GPU: the target of the ncu
-    captures summarized under profiles/ (launch 3 of the fused forward, launch 2 of the
-    calibration SYRK, launch 3 of the decode kernel, the training view's backward
-    products, the NL-MSE launches)."""
+    captures summarized under profiles/ (gpt3_layer: launches 4-6 of tc_gemm_pair_kernel
+    are the three layers' fused forwards, after the three folds; fused: launch 3 of the fused
+    forward at the Llama2 QKV prefill shape; launch 2 of the calibration SYRK; launch 3 of
+    the decode kernel; the training view's backward products; the NL-MSE launches; epilogue:
+    launches 2-3 of a dense 2048 x 6144 x 512 product, a short reduction)."""
     import paper_2410_05437_gb300 as esp
     torch.cuda.set_device(0)
-    if which in ("fused", "decode"):
+    if which == "gpt3_layer":
+        layers = build_layers(esp, synth.BASE_SEED + 800)
+        for l in layers:
+            esp.espace_linear_forward(l["p"], l["X"], l["Y"])
+        torch.cuda.synchronize()
+        for l in layers:
+            esp.espace_proj_destroy(l["p"])
+    elif which == "epilogue":
+        K, M, N = 512, 6144, 2048
+        W = synth.weights_device(M, K)
+        X = synth.ActivationModel(K).sample_device(N)
+        Y = torch.empty(N, M, device="cuda", dtype=torch.bfloat16)
+        for _ in range(3):
+            esp.espace_dense_forward(X, W, Y)
+        torch.cuda.synchronize()
+    elif which in ("fused", "decode"):
         K, M, L = 4096, 12288, 2048
         N = 4096 if which == "fused" else 1
         W = synth.weights_device(M, K)

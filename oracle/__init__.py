@@ -10,7 +10,8 @@ arrays and chains the steps in the order the paper states them:
 * ``autocorr_rows``     the same for selected rows (large K);
 * ``eigh``              the EVD of Sec. 3.1 by cyclic Jacobi, eigenvalues decreasing;
 * ``build_projection``  Thm. 1: P = the L principal eigenvectors of C = S / n, then bf16;
-* ``fold``              W' = P^T W (Sec. 2.2), bf16;
+* ``fold``              W' = P^T W (Sec. 2.2), bf16 (``fold_matmul``: the same with
+  numpy's matrix product as the product step, for full-size layers);
 * ``project``           Z = P^T X, rounded to bf16 (the rank-L intermediate of Eq. 3);
 * ``contract``          Y = W'^T Z (Eq. 3), fp64;
 * ``forward``           project then contract: the projected linear layer of Eq. 3;
@@ -154,6 +155,18 @@ def fold(P, W, round_bf16: bool = True) -> np.ndarray:
     Wf = np.zeros((L, M))
     _load().oracle_fold(_ptr(P), _ptr(W), K, M, L, _ptr(Wf), int(round_bf16))
     return Wf
+
+
+def fold_matmul(P, W, round_bf16: bool = True) -> np.ndarray:
+    """``W' = P^T W`` by the same definition as ``fold``, with numpy's fp64 matrix product
+    (a library primitive) as the product step: the full-size parity tests fold layers of
+    up to 12288 x 24576 x 6144, where the plain loops take many minutes. Only the
+    summation order differs from ``fold`` (fp64 either way); each entry is then rounded to
+    bf16 by the oracle's own rounding."""
+    P, W = _f64(P), _f64(W)
+    assert W.shape[1] == P.shape[0]
+    Wf = np.ascontiguousarray(P.T @ W.T)
+    return bf16_round(Wf) if round_bf16 else Wf
 
 
 def project(X, P, round_bf16: bool = True) -> np.ndarray:

@@ -365,7 +365,9 @@ def test_train_forward_backward_matches_oracle(esp, N, K, M, L):
         assert np.all(Zg[:, L:] == 0)
         assert_close_normwise(Z[:, :L], Z_o)
         assert_y_close(Y, Y_o)
-        dX_o, dW_o = oracle.train_backward(f64(dY), Zg[:, :L], Pb, Wf)
+        # the backward products are checked from the oracle's own Z (the GPU's Z may differ
+        # from it by isolated one-ulp roundings, within the tolerances)
+        dX_o, dW_o = oracle.train_backward(f64(dY), Z_o, Pb, Wf)
         assert_close_normwise(dX, dX_o)
         assert_close_normwise(dW, dW_o)
         # two micro-batches of one step: the weight gradient sums over both (their tokens)
@@ -377,7 +379,8 @@ def test_train_forward_backward_matches_oracle(esp, N, K, M, L):
         esp.espace_train_backward(p, dev(dY2), Z2, dX)
         esp.espace_train_weight_grad(p, dW)
         torch.cuda.synchronize()
-        both = np.concatenate([Zg[:, :L], f64(Z2)[:, :L]])
+        Z2_o = oracle.forward(f64(X2), Pb, f64(W), Wf=Wf)[1]
+        both = np.concatenate([Z_o, Z2_o])
         _, dW_o2 = oracle.train_backward(np.concatenate([f64(dY), f64(dY2)]), both, Pb, Wf)
         assert_close_normwise(dW, dW_o2)
         # an optimizer step: new weights, W' refolded on the device
@@ -594,8 +597,8 @@ def test_build_projection_tp(esp):
 
 @pytest.mark.slow
 def test_llama2_qkv_prefill_full_size_sampled(esp):
-    """K=4096, M=12288, L=2048, N=4096 (the benchmark launch): every output of 66 sampled
-    tokens over 256 sampled output features against the oracle."""
+    """K=4096, M=12288, L=2048, N=4096 (the Llama2 QKV prefill launch): all 12,288 outputs
+    of 66 sampled tokens (the first, the last and 64 seeded ones) against the oracle."""
     K, M, L, N = 4096, 12288, 2048, 4096
     seed = synth.config_seed("llama2_qkv_prefill")
     model, X, W = make_layer(K, M, N, seed=seed)
@@ -608,12 +611,11 @@ def test_llama2_qkv_prefill_full_size_sampled(esp):
         esp.espace_check()
         r = np.random.default_rng(seed)
         toks = np.unique(np.concatenate([[0, N - 1], r.choice(N, 64, replace=False)]))
-        cols = np.sort(r.choice(M, 256, replace=False))
         Pb = oracle.bf16_round(P)
-        Wf_o = oracle.fold(Pb, f64(W[cols]))
+        Wf_o = oracle.fold_matmul(Pb, f64(W))
         Z_o = oracle.project(f64(X[toks]), Pb)
         Y_o = oracle.contract(Z_o, Wf_o)
-        assert_y_close(f64(Y[toks][:, cols]), Y_o)
+        assert_y_close(f64(Y[toks]), Y_o)
     finally:
         esp.espace_proj_destroy(p)
 

@@ -284,6 +284,27 @@ def test_fold_project_contract_dense_brute_force():
             assert abs(Yd[t, m] - sum(W[m][k] * X[t][k] for k in range(K))) < 1e-13
 
 
+def test_fold_matmul_matches_the_loop_fold():
+    """The matrix-product fold used at full sizes: brute force on a tiny shape, and the
+    loop fold's bf16 values on a moderate one (same fp64 definition, another summation
+    order: a rounding can differ only where the fp64 sums straddle a tie)."""
+    r = rng(14)
+    K, M, L = 6, 5, 3
+    P, W = r.standard_normal((K, L)), r.standard_normal((M, K))
+    Wf = oracle.fold_matmul(P, W, round_bf16=False)
+    for l in range(L):
+        for m in range(M):
+            assert abs(Wf[l, m] - sum(P[k][l] * W[m][k] for k in range(K))) < 1e-13
+    K, M, L = 384, 200, 96
+    P = oracle.bf16_round(r.standard_normal((K, L)) * K ** -0.5)
+    W = oracle.bf16_round(r.standard_normal((M, K)) * K ** -0.5)
+    a, b = oracle.fold_matmul(P, W), oracle.fold(P, W)
+    assert a.shape == (L, M)
+    assert np.mean(a == b) > 0.9999
+    assert np.all(np.abs(a - b) <= 2.0 ** -7 * np.abs(b))      # at most one bf16 ulp apart
+    assert np.array_equal(oracle.bf16_round(a), a)
+
+
 def test_eq3_associativity():
     """(P^T W)^T (P^T X) = W^T (P P^T X) for non-square shapes."""
     r = rng(13)
