@@ -316,13 +316,19 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
  * 16 MiB, enough for N * Lp <= 8,388,608 (e.g. 4096 tokens at L = 2048). */
 #define ESPACE_NOALLOC_Z_ELEMS 8388608
 
-/* Async. Same result as espace_linear_forward (automatic path) for callers that cannot
+/* Async. The projected forward of espace_linear_forward, equal to it within the parity
+ * tolerances, for callers that cannot
  * allocate device memory during the call -- for example code that runs inside a memory
  * budget or pool owned by someone else, or a server that reserved all device memory at
  * start-up. Instead of the handle's growable Z scratch it uses one fixed array of
  * ESPACE_NOALLOC_Z_ELEMS bf16 values that is part of the library image on every device
  * that loads the library (held until the process exits); the call itself allocates
  * nothing. The paper has no counterpart: it is an interface convenience of this library.
+ *   - Kernels: the decode kernel for N <= 32 when the layer fits it (the automatic path
+ *     takes it only up to 16 tokens), else one tcgen05 launch per product with Z through
+ *     the fixed array (the automatic path may instead run both products in one launch, or
+ *     split a reduction over the SMs); results can differ from espace_linear_forward's in
+ *     the last bf16 bit, and the speed differs.
  *   - N * Lp (Lp = L rounded up to a multiple of 64) above ESPACE_NOALLOC_Z_ELEMS is
  *     rejected with ESPACE_ERR_SHAPE before anything is launched.
  *   - The handle's device must be current (ESPACE_ERR_STATE otherwise).
@@ -365,6 +371,11 @@ int espace_set_wait_limit_ns(uint64_t ns);
  * nothing completes, gives up after limit_ns (at most 1e9) and records ESPACE_ERR_TIMEOUT,
  * so that the next espace_check() reports it. Nothing faults and the context stays usable. */
 int espace_debug_wait_timeout(uint64_t limit_ns, void* stream);
+
+/* Test hook for persistent kernels sharing the GPU: launches (async) `ctas` CTAs (1 .. the
+ * SM count), each holding one SM with 200 KB of shared memory for hold_ns (at most 1e9),
+ * so that a kernel launched meanwhile on another stream finds only the other SMs free. */
+int espace_debug_occupy(int ctas, uint64_t hold_ns, void* stream);
 
 /* ---------------------------------------------------------------------------------------
  * Host-only helper (no GPU needed)

@@ -30,7 +30,7 @@ __all__ = [
     "espace_proj_export", "espace_proj_import", "espace_proj_destroy",
     "espace_linear_forward", "espace_linear_forward_path", "espace_linear_forward_noalloc",
     "espace_dense_forward",
-    "espace_check", "espace_debug_wait_timeout", "espace_set_wait_limit_ns", "espace_set_phase_event",
+    "espace_check", "espace_debug_wait_timeout", "espace_debug_occupy", "espace_set_wait_limit_ns", "espace_set_phase_event",
     "espace_host_eigh",
     "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "PATH_TENSOR_SPLIT", "EXPORTED_SYMBOLS",
     "TP_COLUMN", "TP_ROW", "espace_proj_tp_from_host", "espace_build_projection_tp", "espace_proj_tp_info",
@@ -109,6 +109,7 @@ _SIGNATURES = {
     "espace_dense_backward": (ctypes.c_int, [_vp, _i64, _vp, _i64, _vp, _i64, _vp, _vp, ctypes.c_int, _vp]),
     "espace_check": (ctypes.c_int, [_vp]),
     "espace_debug_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _vp]),
+    "espace_debug_occupy": (ctypes.c_int, [ctypes.c_int, ctypes.c_uint64, _vp]),
     "espace_set_wait_limit_ns": (ctypes.c_int, [ctypes.c_uint64]),
     "espace_set_phase_event": (ctypes.c_int, [_vp]),
     "espace_host_eigh": (ctypes.c_int, [_pd, _i64, _pd, _pd, ctypes.c_int]),
@@ -189,6 +190,10 @@ def espace_check(stream=None) -> None:
 
 def espace_debug_wait_timeout(limit_ns: int, stream=None) -> None:
     _check(lib.espace_debug_wait_timeout(int(limit_ns), _stream(stream)))
+
+
+def espace_debug_occupy(ctas: int, hold_ns: int, stream=None) -> None:
+    _check(lib.espace_debug_occupy(int(ctas), int(hold_ns), _stream(stream)))
 
 
 def espace_host_eigh(A: np.ndarray, threads: int = 0, vectors: bool = True):

@@ -139,12 +139,15 @@ __device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned* p)
 }
 
 // Grid barrier over all CTAs of a cooperative launch, by one thread per CTA; `start` is the
-// counter as this thread read it when the CTA started. Returns false (recording a timeout)
-// if the others did not arrive within the limit.
-__device__ bool grid_arrive_and_wait(unsigned* bar, unsigned start, int* status, uint64_t limit_ns)
+// counter as this thread read it when the CTA started. Every CTA arrives exactly once per
+// launch, also one that has given up (skip_wait), so that the counter's bit flips once per
+// launch and the next launch starts from a consistent count. Returns false (recording a
+// timeout) if the others did not arrive within the limit, or at once with skip_wait.
+__device__ bool grid_arrive_and_wait(unsigned* bar, unsigned start, int* status, uint64_t limit_ns, bool skip_wait)
 {
     const unsigned nb = blockIdx.x == 0 ? 0x80000000u - (gridDim.x - 1) : 1u;
     asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(bar), "r"(nb) : "memory");
+    if (skip_wait) return false;
     const uint64_t t0 = globaltimer_ns();
     uint32_t spins = 0;
     while (((start ^ ld_acquire_gpu(bar)) & 0x80000000u) == 0) {
@@ -415,7 +418,7 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
             volatile int never = 0;
             for (int q = max(0, j - a.stages); q < j; ++q)
                 mbar_wait(&full[q % a.stages], static_cast<uint32_t>(q / a.stages) & 1u, &never, a.status,
-                          a.wait_limit_ns, ESPACE_ERR_TIMEOUT);
+                          cleanup_limit(a.wait_limit_ns), ESPACE_ERR_TIMEOUT);
         }
         return;
     }
@@ -495,11 +498,16 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
         if (p + 1 < a.phases) {
             // every Z of this CTA is stored (consumer_sync above); wait for all CTAs
             if (threadIdx.x == 0) {
-                const bool ok = !*abort && grid_arrive_and_wait(a.bar, bar_start, a.status, a.wait_limit_ns);
+                const bool ok = grid_arrive_and_wait(a.bar, bar_start, a.status, a.wait_limit_ns, *abort != 0);
                 if (!ok) *abort = 1;
             }
         }
         consumer_sync();
+    }
+    if (threadIdx.x == 0 && *abort) {
+        // copies the producer issued before the abort may still be landing in the ring
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 200000ull) __nanosleep(1000);
     }
 }
 

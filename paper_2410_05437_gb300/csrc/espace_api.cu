@@ -10,6 +10,7 @@
 #include <algorithm>
 #include <cmath>
 #include <atomic>
+#include <functional>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -19,6 +20,9 @@
 
 namespace espace {
 int host_eigh(const double* A, int64_t n, double* w, double* V, int threads);
+int host_eigh_select(const double* A, int64_t n, double* w,
+                     const std::function<std::vector<int64_t>(const std::vector<double>&)>& order_sel,
+                     std::vector<double>& V, int threads);
 }
 
 using namespace espace;
@@ -108,6 +112,33 @@ uint16_t bf16_from_double(double x)
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
+// The build's eigen-solve: all K eigenvalues of C (K x K, row-major) in the projection's
+// order into w, and the first L eigenvectors in that order as the columns of P (K x L,
+// row-major). The order is decreasing eigenvalue, or decreasing |eigenvalue| (ties keep the
+// signed order) when by_magnitude is set or C is not positive semidefinite (smallest
+// eigenvalue below -1e-6 of the largest magnitude), as the paper orders an indefinite C.
+// Only those L eigenvectors are formed.
+int principal_eigenvectors(const double* C, int64_t K, int64_t L, bool by_magnitude, std::vector<double>& w,
+                           std::vector<double>& P)
+{
+    std::vector<double> desc(K);
+    std::vector<int64_t> order;
+    auto sel = [&](const std::vector<double>& wd) {
+        order.resize(K);
+        for (int64_t i = 0; i < K; ++i) order[i] = i;
+        const double wmax = std::max(std::fabs(wd[0]), std::fabs(wd[K - 1]));
+        if (by_magnitude || wd[K - 1] < -1e-6 * wmax)
+            std::stable_sort(order.begin(), order.end(),
+                             [&](int64_t a, int64_t b) { return std::fabs(wd[a]) > std::fabs(wd[b]); });
+        return std::vector<int64_t>(order.begin(), order.begin() + L);
+    };
+    const int rc = host_eigh_select(C, K, desc.data(), sel, P, 0);
+    if (rc != ESPACE_OK) return rc;
+    w.resize(K);
+    for (int64_t i = 0; i < K; ++i) w[i] = desc[order[i]];
+    return ESPACE_OK;
+}
+
 }  // namespace
 
 // ============================================================================ device state
@@ -187,7 +218,7 @@ struct espace_proj_s {
     uint16_t* Z = nullptr;         // [zcap][Lp] bf16 scratch for the rank-L intermediate
     int64_t zcap = 0;
     unsigned int* bar = nullptr;   // grid barrier counter of the decode kernel (zeroed)
-    int* ready = nullptr;          // fused forward: 2 x ceil(zcap / 256) zeroed counters
+    int* ready = nullptr;          // fused forward: ceil(zcap / 256) readiness counters, ticket, exit counter (zeroed)
     float* part = nullptr;         // split reductions of the few-token products (fp32)
     int64_t part_cap = 0;
     // tensor-parallel layer (tp_kind != 0): Lp = tp * L is the width of Z. COLUMN: PT is
@@ -588,22 +619,14 @@ int espace_build_projection_go(espace_calib_t h, const void* W_dev, int64_t M, i
     // T = C_X C_W in fp64; C = T + T^T = C_X C_W + C_W C_X (both factors symmetric)
     CUDA_TRY(launch_gemm_f64(cx.as<double>(), cw.as<double>(), static_cast<int>(K), t.as<double>(), st),
              "build_projection_go: product");
-    std::vector<double> T(kk), C(kk), w(K), V(kk);
+    std::vector<double> T(kk), C(kk), wo, P;
     CUDA_TRY(cudaStreamSynchronize(st), "build_projection_go: sync");
     CUDA_TRY(cudaMemcpy(T.data(), t.ptr, sizeof(double) * kk, cudaMemcpyDeviceToHost), "build_projection_go: read");
     for (int64_t i = 0; i < K; ++i)
         for (int64_t j = 0; j < K; ++j) C[i * K + j] = T[i * K + j] + T[j * K + i];
-    rc = host_eigh(C.data(), K, w.data(), V.data(), 0);
-    if (rc != ESPACE_OK) return fail(rc, "espace_build_projection_go: eigen-solver did not converge");
     // C may be indefinite: order by |eigenvalue|, largest first (ties keep the signed order)
-    std::vector<int64_t> order(K);
-    for (int64_t i = 0; i < K; ++i) order[i] = i;
-    std::stable_sort(order.begin(), order.end(),
-                     [&](int64_t a, int64_t b) { return std::fabs(w[a]) > std::fabs(w[b]); });
-    std::vector<double> P(static_cast<size_t>(K * L)), wo(K);
-    for (int64_t i = 0; i < K; ++i) wo[i] = w[order[i]];
-    for (int64_t k = 0; k < K; ++k)
-        for (int64_t l = 0; l < L; ++l) P[k * L + l] = V[k * K + order[l]];
+    rc = principal_eigenvectors(C.data(), K, L, true, wo, P);
+    if (rc != ESPACE_OK) return fail(rc, "espace_build_projection_go: eigen-solver did not converge");
     espace_proj_s* p = nullptr;
     rc = proj_create(K, M, L, &p);
     if (rc != ESPACE_OK) return rc;
@@ -660,23 +683,12 @@ int espace_build_projection(espace_calib_t h, const void* W_dev, int64_t M, int6
     std::vector<float> S;
     rc = read_sum(h, S, stream);
     if (rc != ESPACE_OK) return rc;
-    std::vector<double> C(static_cast<size_t>(K * K)), w(K), V(static_cast<size_t>(K * K));
+    std::vector<double> C(static_cast<size_t>(K * K)), w, P;
     mirror_scaled(S, K, 1.0 / static_cast<double>(h->n), C.data());
-    rc = host_eigh(C.data(), K, w.data(), V.data(), 0);
-    if (rc != ESPACE_OK) return fail(rc, "espace_build_projection: eigen-solver did not converge");
     // decreasing eigenvalues; when C is not positive semidefinite (e.g. an NL-MSE matrix),
-    // decreasing |eigenvalue| instead, as the paper does (ties keep the signed order)
-    std::vector<int64_t> order(K);
-    for (int64_t i = 0; i < K; ++i) order[i] = i;
-    const double wmax = std::max(std::fabs(w[0]), std::fabs(w[K - 1]));
-    if (w[K - 1] < -1e-6 * wmax)
-        std::stable_sort(order.begin(), order.end(),
-                         [&](int64_t a, int64_t b) { return std::fabs(w[a]) > std::fabs(w[b]); });
-    std::vector<double> P(static_cast<size_t>(K * L)), wo(K);
-    for (int64_t i = 0; i < K; ++i) wo[i] = w[order[i]];
-    w = wo;
-    for (int64_t k = 0; k < K; ++k)
-        for (int64_t l = 0; l < L; ++l) P[k * L + l] = V[k * K + order[l]];
+    // decreasing |eigenvalue| instead, as the paper does
+    rc = principal_eigenvectors(C.data(), K, L, false, w, P);
+    if (rc != ESPACE_OK) return fail(rc, "espace_build_projection: eigen-solver did not converge");
     espace_proj_s* p = nullptr;
     rc = proj_create(K, M, L, &p);
     if (rc != ESPACE_OK) return rc;
@@ -801,15 +813,14 @@ int espace_build_projection_tp(espace_calib_t h, const void* W_dev, int64_t M, i
     mirror_scaled(S, K, 1.0 / static_cast<double>(h->n), C.data());
     const int64_t Kr = K / tp;
     std::vector<double> P(static_cast<size_t>(tp * Kr * L)), evals(static_cast<size_t>(K));
-    std::vector<double> Cr(static_cast<size_t>(Kr * Kr)), w(Kr), V(static_cast<size_t>(Kr * Kr));
+    std::vector<double> Cr(static_cast<size_t>(Kr * Kr)), w, Pr;
     for (int r = 0; r < tp; ++r) {
         // rank r's inputs are features r Kr .. (r+1) Kr: its autocorrelation is C's diagonal block
         for (int64_t i = 0; i < Kr; ++i)
             for (int64_t j = 0; j < Kr; ++j) Cr[i * Kr + j] = C[(r * Kr + i) * K + r * Kr + j];
-        rc = host_eigh(Cr.data(), Kr, w.data(), V.data(), 0);
+        rc = principal_eigenvectors(Cr.data(), Kr, L, false, w, Pr);
         if (rc != ESPACE_OK) return fail(rc, "espace_build_projection_tp: eigen-solver did not converge");
-        for (int64_t k = 0; k < Kr; ++k)
-            for (int64_t l = 0; l < L; ++l) P[(r * Kr + k) * L + l] = V[k * Kr + l];
+        std::copy(Pr.begin(), Pr.end(), P.begin() + r * Kr * L);
         for (int64_t i = 0; i < Kr; ++i) evals[r * Kr + i] = w[i];
     }
     espace_proj_s* p = nullptr;
@@ -956,9 +967,11 @@ static int ensure_z(espace_proj_s* p, int64_t N, cudaStream_t st)
     p->zcap = 0;
     const int64_t cap = std::max<int64_t>(N, 128);
     cudaError_t e = cudaMalloc(&p->Z, sizeof(uint16_t) * cap * p->Lp);
+    // fused forward: one readiness counter per 256-row block of Z, then its work-item
+    // ticket and exit counter
     const int64_t blocks = (cap + 255) / 256;
-    if (e == cudaSuccess) e = cudaMalloc(&p->ready, sizeof(int) * 2 * blocks);
-    if (e == cudaSuccess) e = cudaMemset(p->ready, 0, sizeof(int) * 2 * blocks);
+    if (e == cudaSuccess) e = cudaMalloc(&p->ready, sizeof(int) * (blocks + 2));
+    if (e == cudaSuccess) e = cudaMemset(p->ready, 0, sizeof(int) * (blocks + 2));
     if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "forward: Z scratch of %lld tokens: %s", (long long)cap, cudaGetErrorString(e));
     p->zcap = cap;
     return ESPACE_OK;
@@ -1444,6 +1457,19 @@ int espace_debug_wait_timeout(uint64_t limit_ns, void* stream)
     if (limit_ns == 0 || limit_ns > 1000000000ull)
         return fail(ESPACE_ERR_ARG, "espace_debug_wait_timeout: limit must be in (0, 1e9] ns");
     CUDA_TRY(launch_wait_timeout(limit_ns, static_cast<cudaStream_t>(stream)), "espace_debug_wait_timeout");
+    return ESPACE_OK;
+}
+
+int espace_debug_occupy(int ctas, uint64_t hold_ns, void* stream)
+{
+    DeviceInfo* dev = nullptr;
+    int rc = device_info(&dev);
+    if (rc != ESPACE_OK) return rc;
+    if (ctas < 1 || ctas > dev->num_sms)
+        return fail(ESPACE_ERR_ARG, "espace_debug_occupy: ctas must be in [1, %d]", dev->num_sms);
+    if (hold_ns == 0 || hold_ns > 1000000000ull)
+        return fail(ESPACE_ERR_ARG, "espace_debug_occupy: hold must be in (0, 1e9] ns");
+    CUDA_TRY(launch_occupy(ctas, hold_ns, static_cast<cudaStream_t>(stream)), "espace_debug_occupy");
     return ESPACE_OK;
 }
 

@@ -25,11 +25,13 @@ cudaError_t launch_gemm_tn(const void* A, int64_t lda, const void* B, int64_t ld
                            int cols, int kdim, void* C, int64_t ldc, cudaStream_t stream);
 
 // The projected forward Z = X P, Y = Z W' in one persistent launch of the CTA-pair kernel:
-// Z tiles first, then Y tiles; a Y tile's producer waits (bounded) until the 256-row block
-// of Z it reads is complete. ready / done: ceil(N / 256) zeroed ints each, owned by the
-// caller, left zeroed again by the kernel. Needs N, Lp > 128 to be worthwhile.
+// work items drawn from an atomic ticket, Z tiles first, then Y tiles; a Y tile's producer
+// waits (bounded) until the 256-row block of Z it reads is complete. ready: ceil(N / 256)
+// zeroed ints, sched: two zeroed ints (ticket, exit counter), owned by the caller; the last
+// CTA to leave zeroes them again, also after a launch that gave up waiting. One launch at
+// a time may use them. Needs N, Lp > 128 to be worthwhile.
 cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,
-                                 int K, int Lp, int M, int* ready, int* done, cudaStream_t stream);
+                                 int K, int Lp, int M, int* ready, int* sched, cudaStream_t stream);
 
 // Swapped product: out[n][r] (bf16, leading dimension ldo) = sum_k W[r][k] X[n][k], the
 // weights as the 128-row tcgen05 operand, the tile stored transposed, token tiles of 128
@@ -112,6 +114,8 @@ cudaError_t launch_normalize_rows(const void* X, int64_t N, int K, void* Xn, cud
 // One thread waits on an mbarrier that never completes; after limit_ns it records
 // ESPACE_ERR_TIMEOUT in the status word and returns.
 cudaError_t launch_wait_timeout(uint64_t limit_ns, cudaStream_t stream);
+// `ctas` CTAs that each hold one SM (200 KB of shared memory) for hold_ns, then leave.
+cudaError_t launch_occupy(int ctas, uint64_t hold_ns, cudaStream_t stream);
 
 // C[K][K] (fp64) = scale * (the symmetric matrix whose upper triangle is Su, fp32).
 cudaError_t launch_sym_full_f64(const float* Su, int64_t K, double scale, double* C, cudaStream_t stream);

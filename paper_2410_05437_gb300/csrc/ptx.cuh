@@ -64,6 +64,43 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity)
     return ok != 0;
 }
 
+// As mbar_try_wait with acquire semantics at cluster scope: the waiter then sees what the
+// arriving thread of either CTA of the cluster wrote before a release.cluster arrive.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n"
+        " .reg .pred p;\n"
+        " mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n"
+        "}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait as mbar_wait, with cluster-scope acquire (mbar_try_wait_cluster).
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                                  int* status, uint64_t limit_ns, int code)
+{
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    uint64_t t0 = globaltimer_ns();
+    uint32_t spins = 0;
+    while (!mbar_try_wait_cluster(bar, parity)) {
+        if ((++spins & 63u) == 0) {
+            if (*abort) return false;
+            if (globaltimer_ns() - t0 > limit_ns) {
+                *abort = 1;
+                atomicExch(status, code);
+                return false;
+            }
+        }
+    }
+    return true;
+}
+
 // Waits for the phase of `bar` with the given parity to complete. Gives up (returning
 // false) when *abort is set by another thread of the CTA, or after `limit_ns` of waiting,
 // in which case it sets *abort, records `code` in the device status word and returns false.
@@ -84,6 +121,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
         }
     }
     return true;
+}
+
+// Limit of the waits that clean up after a role gave up (in-flight copies landing, issued
+// MMAs completing): these always end by themselves within microseconds, so they never
+// take the caller's limit when it is shorter than this.
+constexpr uint64_t CLEANUP_WAIT_NS = 100000000ull;
+
+__device__ __forceinline__ uint64_t cleanup_limit(uint64_t limit_ns)
+{
+    return limit_ns > CLEANUP_WAIT_NS ? limit_ns : CLEANUP_WAIT_NS;
 }
 
 // ------------------------------------------------------------------------------ TMA
@@ -247,6 +294,11 @@ __device__ __forceinline__ uint32_t ld_shared_cluster_u32(uint32_t cluster_addr)
     uint32_t v;
     asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(cluster_addr) : "memory");
     return v;
+}
+
+__device__ __forceinline__ void st_shared_cluster_u32(uint32_t cluster_addr, uint32_t v)
+{
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
 }
 
 // Arrive on an mbarrier given by its shared::cluster address (possibly another CTA's).

@@ -234,7 +234,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             // every MMA issued above has finished once this commit arrives
             umma_commit(drain);
             volatile int never = 0;
-            mbar_wait(drain, 0, &never, args.status, limit, ESPACE_ERR_TIMEOUT);
+            mbar_wait(drain, 0, &never, args.status, cleanup_limit(limit), ESPACE_ERR_TIMEOUT);
         }
     } else {
         // ------------------------------------------------------------ epilogue (4 warps)
@@ -315,6 +315,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 
     __syncwarp();
     tc_fence_before_sync();
+    // a role that gave up may leave copies in flight into shared memory: let them land
+    if (threadIdx.x == 0 && *abort_flag) settle_copies();
     __syncthreads();
     if (warp == 1) {
         tc_fence_after_sync();
@@ -340,7 +342,9 @@ constexpr int PAIR_B_BYTES = 128 * BK * 2;
 constexpr int PAIR_STAGE_BYTES = PAIR_A_BYTES + PAIR_B_BYTES;
 constexpr int PAIR_ACCS = 2;        // TMEM accumulators per CTA (1 or 2)
 constexpr int PAIR_TMEM_COLS = PAIR_ACCS * PAIR_BN;
-constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 256;
+// Work items in flight between the leader's producer and the other roles (see PairArgs).
+constexpr int PAIR_RING = 16;
+constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 512;
 // The autocorrelation restarts its TMEM accumulator every SYRK_CHUNK k-blocks (1024
 // tokens) and its epilogue adds the chunks in fp32 registers, so that long token runs do
 // not lose precision in the tensor core's accumulator.
@@ -375,9 +379,17 @@ struct PairProblem {
 // output (the projected layer: Z = X P, then Y = Z W'). Row block tm of the second
 // product's A is read only after both CTAs of every tile in row block tm of the first
 // product have stored it: ready[tm] counts the epilogue warps that stored their rows
-// (target 8 x tiles_n of product 0: four warps in each of two CTAs per tile);
-// done[tm] counts the second product's producers that passed the check, and the last one
-// resets both, so the counters are zero again for the next launch.
+// (target 8 x tiles_n of product 0: four warps in each of two CTAs per tile).
+//
+// Work items: the leader CTA's producer draws them and hands each to every role of both
+// CTAs through a ring in shared memory. With a ticket counter (the two-product program)
+// the items are drawn from it with atomics, so they start in one global order, first
+// product first, and only pairs that are running draw any: a pair that draws a tile of
+// the second product knows that every tile of the first was drawn by a running pair, so
+// its wait ends even when some CTA pairs of the grid are not resident (SMs held by other
+// work). Without a ticket a pair takes items pair, pair + npairs, ... The last CTA to
+// leave (exit counter) zeroes ready[0 .. nready), the ticket and the exit counter, on
+// every exit path, so the next launch starts from zero even after one that gave up.
 //
 // Block-diagonal product (problem 0 of a one-product program, nblocks > 0): output column
 // block g, columns [c0[g], c0[g] + cw[g]), is A[:, ak0[g] .. ak0[g] + kdim) times rows
@@ -389,7 +401,9 @@ struct PairArgs {
     PairProblem p[2];
     int nprob;
     int* ready;
-    int* done;
+    int nready;
+    int* ticket;      // work-item ticket, or nullptr for the static order
+    int* exit_ctr;    // CTAs that left (with a ticket)
     int* status;
     uint64_t wait_limit_ns;
     int nblocks;
@@ -548,7 +562,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
     uint64_t* tfull = empty + PAIR_STAGES;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* ring_full = drain + 1;
+    uint64_t* ring_empty = ring_full + PAIR_RING;
+    int* ring_item = reinterpret_cast<int*>(ring_empty + PAIR_RING);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ring_item + PAIR_RING);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -568,6 +585,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
             mbar_init(&tempty[a], 2 * 32 * PairShape<SYRK>::EPI_WARPS);   // both CTAs' epilogues
         }
         mbar_init(drain, 1);
+        for (int s = 0; s < PAIR_RING; ++s) {
+            mbar_init(&ring_full[s], 1);
+            // the leader's MMA issuer and epilogue warps, the peer's producer and epilogue warps
+            mbar_init(&ring_empty[s], 2 + 2 * PairShape<SYRK>::EPI_WARPS);
+        }
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -594,13 +616,58 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
         tmem_agree ? pair_items(args.p[0]) + (args.nprob > 1 ? pair_items(args.p[1]) : 0) : 0;
     const uint64_t limit = args.wait_limit_ns;
 
+    // i-th work item of this pair (leader's producer only): -1 when there is none left
+    auto draw = [&](int i) -> int {
+        const int it = args.ticket != nullptr ? atomicAdd(args.ticket, 1) : pair + i * npairs;
+        return it < num_items ? it : -1;
+    };
+    // the i-th item from this CTA's ring; false if the wait gave up
+    auto take_item = [&](int i, int& item) -> bool {
+        const int idx = i % PAIR_RING;
+        if (!mbar_wait_cluster(&ring_full[idx], static_cast<uint32_t>(i / PAIR_RING) & 1u, abort_flag,
+                               args.status, limit, ESPACE_ERR_TIMEOUT))
+            return false;
+        item = *reinterpret_cast<volatile int*>(&ring_item[idx]);
+        return true;
+    };
+    // frees ring slot i for the leader's producer
+    auto release_item = [&](int i) {
+        mbar_arrive_cluster(mapa_shared(smem_u32(&ring_empty[i % PAIR_RING]), 0));
+    };
+
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer (both CTAs)
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
-            for (int item = pair; ok && item < num_items; item += npairs) {
+            int next = leader ? draw(0) : -1;
+            for (int i = 0; ok; ++i) {
+                int item;
+                if (leader) {
+                    // publish the item to both CTAs' rings once every role has taken the
+                    // slot's previous one
+                    const int idx = i % PAIR_RING;
+                    if (!mbar_wait_cluster(&ring_empty[idx], (static_cast<uint32_t>(i / PAIR_RING) & 1u) ^ 1u,
+                                           abort_flag, args.status, limit, ESPACE_ERR_TIMEOUT)) {
+                        ok = false;
+                        break;
+                    }
+                    item = next;
+                    ring_item[idx] = item;
+                    st_shared_cluster_u32(mapa_shared(smem_u32(&ring_item[idx]), 1), static_cast<uint32_t>(item));
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&ring_full[idx]), 0));
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&ring_full[idx]), 1));
+                    if (item < 0) break;
+                    next = draw(i + 1);   // its latency overlaps this item's loads
+                } else {
+                    if (!take_item(i, item)) {
+                        ok = false;
+                        break;
+                    }
+                    release_item(i);
+                    if (item < 0) break;
+                }
                 int prob, tm, tn, kb0, kb1;
                 pair_decode(args, item, prob, tm, tn, kb0, kb1);
                 const CUtensorMap* ma = prob == 0 ? &map_a0 : &map_a1;
@@ -622,10 +689,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                     }
                     if (!ok) break;
                     fence_proxy_async_global();   // the TMA reads below see those stores
-                    if (atomicAdd(args.done + tm, 1) == 2 * args.p[1].tiles_n - 1) {
-                        atomicExch(args.ready + tm, 0);
-                        atomicExch(args.done + tm, 0);
-                    }
                 }
                 int ak0, brow, ccol, cend;
                 pair_block_of(args, prob, tn, 0, ak0, brow, ccol, cend);
@@ -678,7 +741,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            for (int item = pair; ok && item < num_items; item += npairs) {
+            for (int i = 0; ok; ++i) {
+                int item;
+                if (!take_item(i, item)) break;
+                release_item(i);
+                if (item < 0) break;
                 int prob, tm, tn, kb0, kb1;
                 pair_decode(args, item, prob, tm, tn, kb0, kb1);
                 // one accumulation per item, or per 16-block chunk of it for SYRK
@@ -723,7 +790,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
             }
             umma_commit_pair(drain, 0x1);
             volatile int never = 0;
-            mbar_wait(drain, 0, &never, args.status, limit, ESPACE_ERR_TIMEOUT);
+            mbar_wait(drain, 0, &never, args.status, cleanup_limit(limit), ESPACE_ERR_TIMEOUT);
         }
     } else if (SYRK) {
         // ------------------------------------------------------------ SYRK epilogue (8 warps)
@@ -735,7 +802,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
         int acc = 0;
         uint32_t acc_phase = 0;
         bool ok = true;
-        for (int item = pair; ok && item < num_items; item += npairs) {
+        for (int i = 0; ok; ++i) {
+            int item;
+            if (!take_item(i, item)) break;
+            __syncwarp();
+            if (lane == 0) release_item(i);
+            if (item < 0) break;
             int prob, tm, tn, kb0, kb1;
             pair_decode(args, item, prob, tm, tn, kb0, kb1);
             const PairProblem pb = pair_problem_of(args, prob);
@@ -809,7 +881,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
         const int row_in_tile = static_cast<int>(rank) * 128 + quarter * 32 + lane;
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (int item = pair; item < num_items; item += npairs) {
+        for (int i = 0;; ++i) {
+            int item;
+            if (!take_item(i, item)) break;
+            __syncwarp();
+            if (lane == 0) release_item(i);
+            if (item < 0) break;
             int prob, tm, tn, kb0, kb1;
             pair_decode(args, item, prob, tm, tn, kb0, kb1);
             const PairProblem pb = pair_problem_of(args, prob);
@@ -868,11 +945,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
     }
 
     __syncwarp();
+    // a CTA whose roles gave up may still have copies in flight, into its own shared memory
+    // or signalling its peer's barriers: both CTAs stay until they have landed
+    if (threadIdx.x == 0 && *abort_flag) settle_copies();
     tc_fence_before_sync();
     cluster_sync();   // no CTA leaves while its peer may still touch its barriers or TMEM
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc_pair(tmem_base, PAIR_TMEM_COLS);
+    }
+    if (args.exit_ctr != nullptr && threadIdx.x == 0) {
+        // every thread of this CTA is past its last use of the counters (cluster barrier);
+        // the last CTA of the grid zeroes them for the next launch
+        __threadfence();
+        if (atomicAdd(args.exit_ctr, 1) == static_cast<int>(gridDim.x) - 1) {
+            __threadfence();
+            volatile int* r = args.ready;
+            for (int b = 0; b < args.nready; ++b) r[b] = 0;
+            *reinterpret_cast<volatile int*>(args.ticket) = 0;
+            __threadfence();
+            *reinterpret_cast<volatile int*>(args.exit_ctr) = 0;
+        }
     }
 }
 
@@ -1472,7 +1565,7 @@ cudaError_t launch_gemm_nn(const void* A, int64_t lda, const void* B, int64_t ld
 }
 
 cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const void* WfT, void* Y, int N,
-                                 int K, int Lp, int M, int* ready, int* done, cudaStream_t stream)
+                                 int K, int Lp, int M, int* ready, int* sched, cudaStream_t stream)
 {
     if (N <= 0) return cudaSuccess;
     DeviceInfo* dev = nullptr;
@@ -1487,7 +1580,9 @@ cudaError_t launch_forward_fused(const void* X, const void* PT, void* Z, const v
     a.p[1] = pair_problem(N, M, Lp, Y, M);
     a.nprob = 2;
     a.ready = ready;
-    a.done = done;
+    a.nready = (N + PAIR_BM - 1) / PAIR_BM;
+    a.ticket = sched;
+    a.exit_ctr = sched + 1;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
     return launch_pair<false>(maps, a, dev, stream);

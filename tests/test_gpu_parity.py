@@ -5,6 +5,8 @@ on C = S / n, normwise 1e-5. Z is rounded to bf16 on both sides (fp32 accumulati
 GPU, fp64 in the oracle), so isolated one-ulp flips of Z at rounding ties are expected and
 covered by the Y tolerance.
 """
+import time
+
 import numpy as np
 import pytest
 import torch
@@ -887,3 +889,87 @@ def test_bounded_wait_reports_timeout_and_context_survives(esp):
     esp.espace_dense_forward(X, W, Y)
     torch.cuda.synchronize()
     assert torch.all(Y.float() == 64.0)
+
+
+def _layer_and_reference(esp, K, M, L, N, seed):
+    _, X, W = make_layer(K, M, N, seed=seed)
+    P = synth.random_projection(K, L, seed=seed)
+    p = esp.espace_proj_from_host(P, dev(W))
+    Y_o = oracle.forward(f64(X), oracle.bf16_round(P), f64(W))[0]
+    return p, dev(X), Y_o
+
+
+def test_fused_forward_completes_while_other_work_holds_half_the_sms(esp):
+    """The fused forward's CTA pairs draw their work items from a ticket, Z tiles first: a
+    pair that draws a Y tile waits only for Z tiles already drawn by running pairs. So with
+    half of the SMs held by another stream's kernel (300 ms), the forward runs on the other
+    half within a 50 ms wait limit and gives the right result; with the items split among
+    the pairs in advance, a resident pair would wait for Z tiles of a pair that cannot
+    start, until the limit."""
+    K, M, L, N = 1024, 2048, 512, 2048
+    p, Xd, Y_o = _layer_and_reference(esp, K, M, L, N, seed=77)
+    try:
+        assert esp.espace_linear_forward_launches(p, N) == 1
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, Xd, Y)            # scratch allocated here
+        torch.cuda.synchronize()
+        esp.espace_check()
+        Y.fill_(float("nan"))
+        sms = torch.cuda.get_device_properties(0).multi_processor_count
+        side = torch.cuda.Stream()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        esp.espace_set_wait_limit_ns(50_000_000)
+        try:
+            esp.espace_debug_occupy(sms // 2, 300_000_000, side)
+            time.sleep(0.02)                            # the holding CTAs are resident
+            a.record()
+            esp.espace_linear_forward(p, Xd, Y)
+            b.record()
+            torch.cuda.synchronize()
+        finally:
+            esp.espace_set_wait_limit_ns(4_000_000_000)
+        esp.espace_check()                              # no wait gave up
+        assert a.elapsed_time(b) < 150.0                # it ran beside the holding kernel
+        assert_y_close(Y, Y_o)
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+@pytest.mark.parametrize("N", [2048, 4])
+def test_forward_after_a_launch_that_gave_up(esp, N):
+    """A launch whose waits give up (a 2 us limit) leaves the handle's counters consistent:
+    the fused kernel's last CTA zeroes its readiness counters, ticket and exit counter on
+    every exit path, and every CTA of the decode kernel arrives once at its grid barrier.
+    The timeout is reported, and the next forwards on the same handle are right."""
+    K, M, L = 1024, 2048, 512
+    p, Xd, Y_o = _layer_and_reference(esp, K, M, L, N, seed=78)
+    try:
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, Xd, Y)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        assert_y_close(Y, Y_o)
+        esp.espace_set_wait_limit_ns(2_000)
+        try:
+            esp.espace_linear_forward(p, Xd, Y)
+            torch.cuda.synchronize()
+        finally:
+            esp.espace_set_wait_limit_ns(4_000_000_000)
+        if N > 32:
+            with pytest.raises(esp.EspaceError) as e:
+                esp.espace_check()
+            assert e.value.code == 5
+        else:
+            try:
+                esp.espace_check()
+            except esp.EspaceError as e:                # the short launch may finish in time
+                assert e.code == 5
+        for _ in range(2):
+            Y.fill_(float("nan"))
+            esp.espace_linear_forward(p, Xd, Y)
+            torch.cuda.synchronize()
+            esp.espace_check()
+            assert_y_close(Y, Y_o)
+    finally:
+        esp.espace_proj_destroy(p)

@@ -38,6 +38,7 @@ def close(Y, Y_ref):
 
 @pytest.mark.parametrize("N,K,M,L", [(128, 512, 512, 256),      # tensor-core kernels
                                      (300, 1024, 776, 300),     # ragged, several tiles
+                                     (24, 1024, 768, 512),      # decode kernel here, swapped tcgen05 there
                                      (4, 512, 512, 256)])       # small-N kernels
 def test_noalloc_forward_matches_forward_twice(esp, N, K, M, L):
     model = synth.ActivationModel(K, seed=N + K)
@@ -80,5 +81,38 @@ def test_noalloc_forward_rejects_batches_beyond_the_fixed_scratch(esp):
         torch.cuda.synchronize()
         esp.espace_check()
         assert torch.all(Y[:Nmax] == 0)
+    finally:
+        esp.espace_proj_destroy(p)
+
+
+@pytest.mark.parametrize("N", [512, 24])
+def test_noalloc_forward_leaves_device_memory_unchanged(esp, N):
+    """The call allocates nothing: with the library's kernels and the fixed array already
+    loaded (a first call), a call on a fresh handle, at a batch size that handle never saw,
+    leaves the device's free memory exactly as it was."""
+    K, M, L = 1024, 1024, 512
+    W = synth.weights(M, K, seed=5).cuda()
+    P = synth.random_projection(K, L, seed=5)
+    X = synth.ActivationModel(K, seed=5).sample(N).cuda()
+    Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+    warm = esp.espace_proj_from_host(P, W)
+    try:
+        esp.espace_linear_forward_noalloc(warm, X[:N // 2].contiguous(), Y[:N // 2])
+        torch.cuda.synchronize()
+    finally:
+        esp.espace_proj_destroy(warm)
+    p = esp.espace_proj_from_host(P, W)
+    try:
+        torch.cuda.synchronize()
+        free0, _ = torch.cuda.mem_get_info()
+        esp.espace_linear_forward_noalloc(p, X, Y)
+        torch.cuda.synchronize()
+        free1, _ = torch.cuda.mem_get_info()
+        esp.espace_check()
+        assert free1 == free0
+        Y_ref = torch.empty_like(Y)
+        esp.espace_linear_forward(p, X, Y_ref)
+        torch.cuda.synchronize()
+        assert close(Y, Y_ref)
     finally:
         esp.espace_proj_destroy(p)
