@@ -48,9 +48,8 @@ SETS = 4
 # over the three layers' launches, from one ncu capture of dram__bytes_read.sum and
 # dram__bytes_write.sum (the gpt3_22b_layer profile case); None until captured for the
 # kernel build that runs.
-FUSED_LAYER_TRAFFIC_BYTES = (1551282176 + 677442816 + 1838649856 + 876077824 + 21090510848 + 594709504) / 3
-FUSED_LAYER_TRAFFIC_SOURCE = ("ncu dram__bytes_read.sum + dram__bytes_write.sum of launches 4-6 of tc_gemm_pair_kernel "
-                              "in bench.py --profile-case gpt3_layer (QKV 2.23, FC1 2.71, FC2 21.69 GB)")
+FUSED_LAYER_TRAFFIC_BYTES = None
+FUSED_LAYER_TRAFFIC_SOURCE = None
 
 
 def parse():
@@ -60,7 +59,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-rows", action="store_true", help="skip the side measurements")
-    ap.add_argument("--profile-case", choices=["gpt3_layer", "fused", "syrk", "decode", "train", "nl", "epilogue"],
+    ap.add_argument("--profile-case", choices=["gpt3_layer", "fused", "split", "syrk", "decode", "train", "nl", "epilogue"],
                     help="run a few launches of one kernel on a fixed case (for ncu) and exit")
     return ap.parse_args()
 
@@ -577,8 +576,8 @@ def config_rows(esp, peak_tc, peak_hbm):
     """(name, row) pairs of the other workloads of the benchmark: the Llama2-7B MLP over a
     rank sweep, calibration over 1,048,576 tokens at K = 6144 and K = 24576, the decode sweep
     on the other Llama2-7B layers, the whole Llama2-7B layer at batch 1, sequence 4096,
-    Table 2's folded tensor-parallel layers (one row per model), the NL-MSE calibration and
-    the training step."""
+    Table 2's folded tensor-parallel layers (one row per model), the NL-MSE calibration, the
+    projection build at K = 4096, 6144 and 11008, and the training step."""
     rows = []
     seed = synth.BASE_SEED + 500
     for name, (K, M) in (("gate_up", (4096, 22016)), ("down", (11008, 4096))):
@@ -620,9 +619,34 @@ def config_rows(esp, peak_tc, peak_hbm):
     for model, r in table2_rows(esp, peak_tc).items():
         rows.append((f"table2_tp_folded_{model}", r))
     rows.append(("nl_mse_calibration", nl_mse_row(esp, peak_tc, seed)))
+    for K, M in ((4096, 12288), (6144, 18432), (11008, 4096)):
+        rows.append((f"build_projection_k{K}", build_row(esp, K, M, K // 2, seed)))
     for name, r in training_rows(esp, peak_tc, seed).items():
         rows.append((f"training_step_{name}", r))
     return rows
+
+
+def build_row(esp, K, M, L, seed, n_cal=65536):
+    """espace_build_projection's wall time (synchronous: fp64 eigen-solve of C on the host
+    cores, P rounded to bf16 and W' = P^T W folded on the GPU) after a calibration of n_cal
+    tokens, at rank L of K inputs and M outputs (Thm. 1, App. B.1)."""
+    X = synth.ActivationModel(K, seed=seed).sample_device(n_cal, stream="calib_tokens")
+    W = synth.weights_device(M, K, seed=seed)
+    h = esp.espace_calib_create(K)
+    p = None
+    try:
+        esp.espace_calib_accumulate(h, X)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        p = esp.espace_build_projection(h, W, L)
+        build_s = time.perf_counter() - t0
+        esp.espace_check()
+    finally:
+        if p:
+            esp.espace_proj_destroy(p)
+        esp.espace_calib_destroy(h)
+    del X, W
+    return {"K": K, "M": M, "L": L, "calib_tokens": n_cal, "build_s": build_s, "host_cores": os.cpu_count()}
 
 
 def nl_mse_row(esp, peak_tc, seed, K=4096, T=4096, reps=4):
@@ -724,7 +748,8 @@ def profile_case(which):
     """A few launches of one kernel, with little else on the GPU: the target of the ncu
     captures summarized under profiles/ (gpt3_layer: launches 4-6 of tc_gemm_pair_kernel
     are the three layers' fused forwards, after the three folds; fused: launch 3 of the fused
-    forward at the Llama2 QKV prefill shape; launch 2 of the calibration SYRK; launch 3 of
+    forward at the Llama2 QKV prefill shape; split: the same forward as two launches per call
+    (launches 2-7 of the kernel); launch 2 of the calibration SYRK; launch 3 of
     the decode kernel; the training view's backward products; the NL-MSE launches; epilogue:
     launches 2-3 of a dense 2048 x 6144 x 512 product, a short reduction)."""
     import paper_2410_05437_gb300 as esp
@@ -744,15 +769,16 @@ def profile_case(which):
         for _ in range(3):
             esp.espace_dense_forward(X, W, Y)
         torch.cuda.synchronize()
-    elif which in ("fused", "decode"):
+    elif which in ("fused", "split", "decode"):
         K, M, L = 4096, 12288, 2048
-        N = 4096 if which == "fused" else 1
+        N = 1 if which == "decode" else 4096
         W = synth.weights_device(M, K)
         p = esp.espace_proj_from_host(synth.random_projection(K, L), W)      # launch 1: fold
         X = synth.ActivationModel(K).sample_device(N)
         Y = torch.empty(N, M, device="cuda", dtype=torch.bfloat16)
+        path = esp.PATH_TENSOR_SPLIT if which == "split" else esp.PATH_AUTO
         for _ in range(3):
-            esp.espace_linear_forward(p, X, Y)
+            esp.espace_linear_forward_path(p, X, Y, path)
         torch.cuda.synchronize()
         esp.espace_proj_destroy(p)
     elif which == "train":

@@ -120,8 +120,9 @@ void espace_calib_destroy(espace_calib_t h);
 
 /* Synchronous. Builds the projected layer from a calibrated accumulator:
  *   1. C = S / n in fp64 on the host;
- *   2. symmetric eigen-decomposition of C in fp64 on the host (Householder
- *      tridiagonalization and implicit QR), eigenvalues sorted decreasing (Sec. 3.1), or
+ *   2. symmetric eigen-decomposition of C in fp64 on the host cores (Householder
+ *      tridiagonalization in panels, divide and conquer on the tridiagonal, only the L
+ *      kept eigenvectors carried back), eigenvalues sorted decreasing (Sec. 3.1), or
  *      by decreasing magnitude when C is not positive semidefinite (smallest eigenvalue
  *      below -1e-6 of the largest magnitude; e.g. an NL-MSE matrix), as the paper does;
  *   3. P = the first L eigenvectors (Thm. 1), each column's largest-magnitude entry made
@@ -381,11 +382,13 @@ int espace_debug_occupy(int ctas, uint64_t hold_ns, void* stream);
  * Host-only helper (no GPU needed)
  * ------------------------------------------------------------------------------------- */
 
-/* fp64 symmetric eigen-decomposition used by espace_build_projection: A_host is K x K
- * row-major symmetric (only read); w receives the eigenvalues in decreasing order and V
- * (K x K row-major, may be NULL) the unit eigenvectors as columns, with the sign
- * convention of espace_build_projection. ESPACE_ERR_NUMERIC if the QR iteration does not
- * converge. Uses up to `threads` host threads (0 = all cores). */
+/* fp64 symmetric eigen-decomposition used by espace_build_projection (panel Householder
+ * tridiagonalization, divide and conquer, compact-WY back-transformation): A_host is
+ * K x K row-major symmetric (only read); w receives the eigenvalues in decreasing order and
+ * V (K x K row-major, may be NULL) the unit eigenvectors as columns, with the sign
+ * convention of espace_build_projection. ESPACE_ERR_NUMERIC if the implicit QR of a small
+ * tridiagonal block does not converge. Uses up to `threads` host threads (0 = all cores;
+ * a positive value sets the OpenMP thread count of the process). */
 int espace_host_eigh(const double* A_host, int64_t K, double* w, double* V, int threads);
 
 #ifdef __cplusplus

@@ -21,6 +21,7 @@
 #include <cuda_runtime.h>
 
 #include <stdlib.h>
+#include <string.h>
 
 #include <algorithm>
 #include <atomic>
@@ -344,7 +345,10 @@ constexpr int PAIR_ACCS = 2;        // TMEM accumulators per CTA (1 or 2)
 constexpr int PAIR_TMEM_COLS = PAIR_ACCS * PAIR_BN;
 // Work items in flight between the leader's producer and the other roles (see PairArgs).
 constexpr int PAIR_RING = 16;
-constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + 512;
+// bf16 epilogue: each warp stages a 32-row x 64-column slice of its tile (4 KB, the
+// 128-byte swizzle of the output tensor map) in one of two buffers and stores it with TMA
+constexpr int PAIR_EPI_BUF = 32 * 128;
+constexpr int PAIR_EPI_BYTES = 4 * 2 * PAIR_EPI_BUF;
 // The autocorrelation restarts its TMEM accumulator every SYRK_CHUNK k-blocks (1024
 // tokens) and its epilogue adds the chunks in fp32 registers, so that long token runs do
 // not lose precision in the tensor core's accumulator.
@@ -359,6 +363,9 @@ template <bool SYRK>
 struct PairShape {
     static constexpr int EPI_WARPS = SYRK ? 8 : 4;   // SYRK: two warps per TMEM lane quarter
     static constexpr int THREADS = 64 + 32 * EPI_WARPS;
+    static constexpr int STAGING = SYRK ? 0 : PAIR_EPI_BYTES;   // epilogue staging (bf16 stores)
+    static constexpr int SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + STAGING + 512;
+    static_assert(SMEM_BYTES <= 232448, "shared memory per CTA");
 };
 
 // One product C[rows][cols] = A[rows][k] B[cols][k]^T of a pair program.
@@ -373,6 +380,8 @@ struct PairProblem {
     // token-reduction (M/N-major) programs: bit 0 = add only column >= row; bit 1 (with
     // ksplit == 1 only) = store the tile instead of adding it
     int upper;
+    // bf16 programs: 1 = store through the output tensor map (TMA), 0 = direct stores
+    int tma_store;
 };
 
 // A program of one product, or of two where the second one's A operand is the first one's
@@ -489,6 +498,7 @@ __device__ __forceinline__ PairProblem pair_problem_of(const PairArgs& a, int pr
     r.out = prob == 0 ? a.p[0].out : a.p[1].out;
     r.ldo = prob == 0 ? a.p[0].ldo : a.p[1].ldo;
     r.upper = prob == 0 ? a.p[0].upper : a.p[1].upper;
+    r.tma_store = prob == 0 ? a.p[0].tma_store : a.p[1].tma_store;
     return r;
 }
 
@@ -552,12 +562,14 @@ template <bool SYRK, bool B_MN = SYRK>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THREADS, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_b0,
                         const __grid_constant__ CUtensorMap map_a1, const __grid_constant__ CUtensorMap map_b1,
+                        const __grid_constant__ CUtensorMap map_c0, const __grid_constant__ CUtensorMap map_c1,
                         const PairArgs args)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + PAIR_STAGES * PAIR_STAGE_BYTES);
+    uint8_t* staging = smem + PAIR_STAGES * PAIR_STAGE_BYTES;   // 1024-byte aligned
+    uint64_t* full = reinterpret_cast<uint64_t*>(staging + PairShape<SYRK>::STAGING);
     uint64_t* empty = full + PAIR_STAGES;
     uint64_t* tfull = empty + PAIR_STAGES;
     uint64_t* tempty = tfull + 2;
@@ -601,6 +613,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
             tma_prefetch_map(&map_a1);
             tma_prefetch_map(&map_b1);
         }
+        if (!SYRK && args.p[0].tma_store) tma_prefetch_map(&map_c0);
+        if (!SYRK && args.nprob > 1 && args.p[1].tma_store) tma_prefetch_map(&map_c1);
     }
     tc_fence_before_sync();
     cluster_sync();   // barriers of both CTAs initialised before any remote arrive or copy
@@ -879,6 +893,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
         // ------------------------------------------------------------ epilogue (both CTAs)
         const int quarter = warp & 3;
         const int row_in_tile = static_cast<int>(rank) * 128 + quarter * 32 + lane;
+        // this warp's two staging buffers (32 rows x 128 bytes each, swizzled as the map's box)
+        uint8_t* stage_buf = staging + quarter * 2 * PAIR_EPI_BUF;
+        uint32_t chunks = 0;   // slices this warp has handed to TMA (buffer = chunks & 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int i = 0;; ++i) {
@@ -899,32 +916,75 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                                    static_cast<uint32_t>(acc * PAIR_BN);
             int ak0, brow, ccol, cend;
             pair_block_of(args, prob, tn, pb.cols, ak0, brow, ccol, cend);
+            if (pb.tma_store) {
+                // 64-column slices: TMEM -> registers -> bf16 in the staging buffer (16-byte
+                // chunk c of row r at chunk c ^ (r % 8)) -> one TMA store per slice, clipped
+                // at the tensor's last row and column
+                const CUtensorMap* mc = prob == 0 ? &map_c0 : &map_c1;
+                const int y0 = tm * PAIR_BM + static_cast<int>(rank) * 128 + quarter * 32;
 #pragma unroll 1
-            for (int c = 0; c < PAIR_BN; c += 32) {
-                const int col0 = ccol + c;
-                if (col0 >= cend) break;             // uniform across the warp
-                uint32_t v[32];
-                tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
-                tmem_ld_wait();
-                if (row >= pb.rows) continue;
-                __nv_bfloat16* out_row =
-                    reinterpret_cast<__nv_bfloat16*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
-                if (col0 + 32 <= cend) {
-                    uint4* dst = reinterpret_cast<uint4*>(out_row + col0);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        uint4 q;
-                        q.x = pack_bf16x2(__uint_as_float(v[8 * i + 0]), __uint_as_float(v[8 * i + 1]));
-                        q.y = pack_bf16x2(__uint_as_float(v[8 * i + 2]), __uint_as_float(v[8 * i + 3]));
-                        q.z = pack_bf16x2(__uint_as_float(v[8 * i + 4]), __uint_as_float(v[8 * i + 5]));
-                        q.w = pack_bf16x2(__uint_as_float(v[8 * i + 6]), __uint_as_float(v[8 * i + 7]));
-                        dst[i] = q;
+                for (int c = 0; c < PAIR_BN; c += 64) {
+                    const int col0 = ccol + c;
+                    if (col0 >= cend) break;             // uniform across the warp
+                    uint8_t* buf = stage_buf + (chunks & 1u) * PAIR_EPI_BUF;
+                    if (chunks >= 2) {
+                        // the store that used this buffer two slices ago has read it
+                        if (lane == 0) bulk_wait_group_read<1>();
+                        __syncwarp();
                     }
-                } else {
+                    uint32_t v[32];
+                    const uint32_t row_addr = smem_u32(buf) + static_cast<uint32_t>(lane) * 128u;
 #pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        if (col0 + i < cend)
-                            out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
+                    for (int h = 0; h < 2; ++h) {
+                        tmem_ld_32cols(t_row + static_cast<uint32_t>(c + 32 * h), v);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            uint4 w;
+                            w.x = pack_bf16x2(__uint_as_float(v[8 * q + 0]), __uint_as_float(v[8 * q + 1]));
+                            w.y = pack_bf16x2(__uint_as_float(v[8 * q + 2]), __uint_as_float(v[8 * q + 3]));
+                            w.z = pack_bf16x2(__uint_as_float(v[8 * q + 4]), __uint_as_float(v[8 * q + 5]));
+                            w.w = pack_bf16x2(__uint_as_float(v[8 * q + 6]), __uint_as_float(v[8 * q + 7]));
+                            const uint32_t chunk = static_cast<uint32_t>((4 * h + q) ^ (lane & 7));
+                            st_shared_v4(row_addr + chunk * 16u, w);
+                        }
+                    }
+                    fence_proxy_async_shared();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(mc, buf, col0, y0);
+                        bulk_commit_group();
+                    }
+                    ++chunks;
+                }
+            } else {
+#pragma unroll 1
+                for (int c = 0; c < PAIR_BN; c += 32) {
+                    const int col0 = ccol + c;
+                    if (col0 >= cend) break;             // uniform across the warp
+                    uint32_t v[32];
+                    tmem_ld_32cols(t_row + static_cast<uint32_t>(c), v);
+                    tmem_ld_wait();
+                    if (row >= pb.rows) continue;
+                    __nv_bfloat16* out_row =
+                        reinterpret_cast<__nv_bfloat16*>(pb.out) + static_cast<int64_t>(row) * pb.ldo;
+                    if (col0 + 32 <= cend) {
+                        uint4* dst = reinterpret_cast<uint4*>(out_row + col0);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            uint4 q;
+                            q.x = pack_bf16x2(__uint_as_float(v[8 * i + 0]), __uint_as_float(v[8 * i + 1]));
+                            q.y = pack_bf16x2(__uint_as_float(v[8 * i + 2]), __uint_as_float(v[8 * i + 3]));
+                            q.z = pack_bf16x2(__uint_as_float(v[8 * i + 4]), __uint_as_float(v[8 * i + 5]));
+                            q.w = pack_bf16x2(__uint_as_float(v[8 * i + 6]), __uint_as_float(v[8 * i + 7]));
+                            dst[i] = q;
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (col0 + i < cend)
+                                out_row[col0 + i] = __float2bfloat16_rn(__uint_as_float(v[i]));
+                    }
                 }
             }
             tc_fence_before_sync();
@@ -935,13 +995,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
             }
             if (prob == 0 && args.nprob > 1 && args.ready != nullptr) {
                 // publish this warp's 32 rows of the tile to the second product's producers
-                // (per warp, so that no block-wide barrier can wait on a warp that gave up)
+                // (per warp, so that no block-wide barrier can wait on a warp that gave up);
+                // TMA stores must have completed, not only read their source
+                if (pb.tma_store && lane == 0) bulk_wait_group<0>();
                 fence_proxy_async_global();
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) red_release_gpu_add(args.ready + tm, 1);
             }
         }
+        // every TMA store of this warp has completed before its staging can go away
+        if (lane == 0) bulk_wait_group<0>();
     }
 
     __syncwarp();
@@ -1053,14 +1117,30 @@ cudaError_t launch_pair(const CUtensorMap* maps, PairArgs& a, const DeviceInfo* 
     const int items = a.p[0].num_tiles * a.p[0].ksplit + (a.nprob > 1 ? a.p[1].num_tiles * a.p[1].ksplit : 0);
     const int pairs = std::min(items, dev->num_sms / 2);
     auto kern = tc_gemm_pair_kernel<SYRK, B_MN>;
+    constexpr int smem = PairShape<SYRK>::SMEM_BYTES;
     static std::atomic<bool> attr_set[64];   // per device; a repeated set is harmless
     if (dev->device < 0 || dev->device >= 64) return cudaErrorInvalidDevice;
     if (!attr_set[dev->device].load(std::memory_order_acquire)) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, PAIR_SMEM_BYTES);
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         attr_set[dev->device].store(true, std::memory_order_release);
     }
-    kern<<<2 * pairs, PairShape<SYRK>::THREADS, PAIR_SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
+    // output tensor maps of the bf16 programs (TMA stores); a problem whose output cannot
+    // be described to TMA (pitch not a multiple of 16 bytes, base not 16-byte aligned) or
+    // that stores only part of its columns (block-diagonal) keeps the direct stores
+    CUtensorMap cmaps[2];
+    memset(cmaps, 0, sizeof(cmaps));
+    for (int q = 0; q < a.nprob && !SYRK; ++q) {
+        PairProblem& pq = a.p[q];
+        pq.tma_store = 0;
+        if (a.nblocks == 0 && pq.cols >= 64 && pq.rows >= 32 && pq.ldo % 8 == 0 &&
+            (reinterpret_cast<uintptr_t>(pq.out) & 15u) == 0 &&
+            encode_map(&cmaps[q], pq.out, pq.cols, pq.rows, pq.ldo, 64, 32))
+            pq.tma_store = 1;
+    }
+    if (a.nprob < 2) cmaps[1] = cmaps[0];
+    kern<<<2 * pairs, PairShape<SYRK>::THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], cmaps[0],
+                                                                  cmaps[1], a);
     return cudaGetLastError();
 }
 

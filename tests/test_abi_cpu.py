@@ -141,3 +141,31 @@ def test_host_eigh_degenerate_and_calibration_spectrum():
     w_o, _, _ = oracle.eigh(S)
     w2 = esp.espace_host_eigh(S, vectors=False)
     assert np.allclose(w2, w_o, rtol=0, atol=1e-12 * w_o[0])
+
+
+@pytest.mark.parametrize("kind", ["graded", "degenerate", "calibration"])
+def test_host_eigh_divide_and_conquer_sizes(kind):
+    """K = 1100: the tridiagonal problem is torn above 512 rows (parallel joins), the panel
+    reduction runs its threaded matrix-vector products. Eigenvalues against LAPACK's (numpy,
+    a test witness), orthogonality and the residual C V = V diag(w) of all K vectors."""
+    import synth
+    import paper_2410_05437_gb300 as esp
+    K = 1100
+    r = np.random.default_rng(11)
+    if kind == "calibration":
+        model = synth.ActivationModel(K, seed=9)
+        X = synth.bf16_to_f64(model.sample(4 * K))
+        C = X.T @ X / (4 * K)
+    else:
+        Q = synth.haar_orthonormal(r, K, K)
+        lam = (np.arange(1, K + 1) ** -1.6 if kind == "graded"
+               else np.repeat(r.standard_normal((K + 7) // 8), 8)[:K])
+        C = (Q * lam) @ Q.T
+        C = (C + C.T) / 2
+    w, V = esp.espace_host_eigh(C)
+    w_ref = np.linalg.eigvalsh(C)[::-1]
+    scale = np.abs(w_ref).max()
+    assert np.all(np.diff(w) <= 0)
+    assert np.allclose(w, w_ref, rtol=0, atol=1e-13 * scale * 10)
+    assert np.abs(V.T @ V - np.eye(K)).max() < 1e-12
+    assert np.abs(C @ V - V * w).max() < 1e-12 * scale

@@ -148,3 +148,53 @@ def test_decode_sweep(esp, layer, N):
     W = synth.weights(M, K, seed=seed)
     P = synth.structured_projection(K, L, seed=seed)
     sampled_check(esp, X, W, P, seed)
+
+
+# ------------------------------------------------------------------ build at a benchmark size (Thm. 1)
+
+def test_build_projection_k4096_from_65536_tokens(esp):
+    """espace_build_projection at the Llama2 QKV shape (K = 4096, L = 2048) from 65,536
+    calibration tokens: C against Eq. 4 (the sum taken with numpy's matrix product as a
+    witness; the oracle's plain loops take minutes here), the eigenvalues against numpy's
+    eigh of that C (a library routine, as a test witness: cyclic Jacobi at K = 4096 is too
+    slow), the well-separated leading eigenvectors one by one, and Thm. 1 for the library's
+    bf16 P: its projection MSE on the calibration tokens is the sum of the discarded
+    eigenvalues (the eigen-gap at L is too small here for a Davis-Kahan bound on P itself)."""
+    K, M, L, n = 4096, 512, 2048, 65536
+    seed = synth.config_seed("llama2_qkv_prefill")
+    X = synth.ActivationModel(K, seed=seed).sample(n, stream="calib_tokens")
+    W = synth.weights(M, K, seed=seed)
+    h = esp.espace_calib_create(K)
+    p = None
+    try:
+        esp.espace_calib_accumulate(h, X.cuda())
+        p = esp.espace_build_projection(h, W.cuda(), L)
+        C, cnt = esp.espace_calib_read(h, K)
+        w = esp.espace_proj_eigenvalues(p)
+        Pb = synth.bf16_to_f64(torch.from_numpy(esp.espace_proj_read_P(p).view(np.int16)).view(torch.bfloat16))
+        esp.espace_check()
+    finally:
+        if p:
+            esp.espace_proj_destroy(p)
+        esp.espace_calib_destroy(h)
+    assert cnt == n
+    Xf = f64(X)
+    C_o = (Xf.T @ Xf) / n
+    del Xf
+    assert np.linalg.norm(C - C_o) / np.linalg.norm(C_o) <= C_REL
+    w_o, V_o = np.linalg.eigh(C_o)
+    w_o, V_o = w_o[::-1], V_o[:, ::-1]
+    assert np.all(np.diff(w) <= 0)
+    assert np.allclose(w, w_o, rtol=0, atol=C_REL * np.linalg.norm(C_o))
+    # leading eigenvectors with relative gaps above 1 %: each column within bf16 rounding
+    for i in range(8):
+        gap = min(w_o[i] - w_o[i + 1], w_o[i - 1] - w_o[i] if i else np.inf) / w_o[0]
+        if gap > 1e-2:
+            assert abs(Pb[:, i] @ V_o[:, i]) / np.linalg.norm(Pb[:, i]) >= 1 - 1e-4, i
+    # Thm. 1: E||x - P P^T x||^2 = tr(C) - 2 tr(P^T C P) + tr(P^T P P^T C P)
+    CP = C_o @ Pb
+    PtP = Pb.T @ Pb
+    mse = np.trace(C_o) - 2 * np.sum(Pb * CP) + np.sum(PtP * (Pb.T @ CP))
+    tail = np.sum(w_o[L:])
+    assert mse <= tail * 1.05 + 1e-3 * np.sum(w_o), (mse, tail)
+    assert mse >= tail * (1 - 1e-6)
