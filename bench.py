@@ -60,7 +60,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-rows", action="store_true", help="skip the side measurements")
-    ap.add_argument("--profile-case", choices=["gpt3_layer", "fused", "split", "syrk", "decode", "train", "nl", "epilogue"],
+    ap.add_argument("--profile-case", choices=["gpt3_layer", "fused", "split", "syrk", "syrk24k", "decode", "train", "nl", "epilogue"],
                     help="run a few launches of one kernel on a fixed case (for ncu) and exit")
     return ap.parse_args()
 
@@ -808,6 +808,15 @@ def profile_case(which):
         h = esp.espace_calib_create(K)
         for _ in range(2):
             esp.espace_calib_accumulate_nl(h, X, G)
+        torch.cuda.synchronize()
+        esp.espace_calib_destroy(h)
+    elif which == "syrk24k":
+        # the calibration SYRK at K = 24576 (FC2's input) over one 16,384-token chunk
+        K, n = 24576, 16384
+        X = synth.ActivationModel(K).sample_device(n, stream="calib_tokens")
+        h = esp.espace_calib_create(K)
+        for _ in range(2):
+            esp.espace_calib_accumulate(h, X)
         torch.cuda.synchronize()
         esp.espace_calib_destroy(h)
     else:
