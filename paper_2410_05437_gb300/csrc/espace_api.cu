@@ -1086,13 +1086,18 @@ int espace_linear_forward_path(espace_proj_t p, const void* X_dev, int64_t N, vo
         // few tokens: the weights are the 128-row operand; phase 1 splits its reduction
         rc = ensure_swap(p, n, dev->num_sms, st);
         if (rc != ESPACE_OK) return rc;
-        CUDA_TRY(launch_gemm_swap(p->PT, K, X_dev, K, Lp, n, K, p->Z, Lp, p->part, st), "forward: phase 1");
+        // both products start streaming the handle's weights (which no kernel of the stream
+        // writes meanwhile) while the grid before them finishes
+        CUDA_TRY(launch_gemm_swap(p->PT, K, X_dev, K, Lp, n, K, p->Z, Lp, p->part, st, mid == nullptr),
+                 "forward: phase 1");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
-        CUDA_TRY(launch_gemm_swap(p->WfT, Lp, p->Z, Lp, M, n, Lp, Y_dev, M, p->part, st), "forward: phase 2");
+        CUDA_TRY(launch_gemm_swap(p->WfT, Lp, p->Z, Lp, M, n, Lp, Y_dev, M, p->part, st, mid == nullptr),
+                 "forward: phase 2");
     } else if (split_phase1_applies(n, K, Lp, M, dev->num_sms, path)) {
         rc = ensure_swap(p, n, dev->num_sms, st);
         if (rc != ESPACE_OK) return rc;
-        CUDA_TRY(launch_gemm_swap(p->PT, K, X_dev, K, Lp, n, K, p->Z, Lp, p->part, st), "forward: phase 1");
+        CUDA_TRY(launch_gemm_swap(p->PT, K, X_dev, K, Lp, n, K, p->Z, Lp, p->part, st, mid == nullptr),
+                 "forward: phase 1");
         if (mid) CUDA_TRY(cudaEventRecord(mid, st), "forward: phase event");
         CUDA_TRY(launch_gemm_tn(p->Z, Lp, p->WfT, Lp, n, M, Lp, Y_dev, M, st), "forward: phase 2");
     } else if (path != ESPACE_PATH_TENSOR_SPLIT && fused_forward_applies(n, Lp, M)) {
@@ -1298,8 +1303,10 @@ int espace_dense_forward(const void* X_dev, int64_t N, int64_t K, const void* W_
             }
             part = ws.part;
         }
+        // like the projected layer's few-token products, it may start loading W while the
+        // grid before it finishes (header: W must not be that grid's output)
         CUDA_TRY(launch_gemm_swap(W_dev, K, X_dev, K, static_cast<int>(M), static_cast<int>(N), static_cast<int>(K), Y_dev,
-                                  M, part, static_cast<cudaStream_t>(stream)),
+                                  M, part, static_cast<cudaStream_t>(stream), true),
                  "espace_dense_forward: launch");
         return ESPACE_OK;
     }

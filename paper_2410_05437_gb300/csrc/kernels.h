@@ -45,8 +45,11 @@ struct SwapPlan {
     int64_t ld_part = 0, part_elems = 0;
 };
 SwapPlan gemm_swap_plan(int rows, int ntok, int kdim, int num_sms, bool allow_split);
+// pdl: launched with programmatic stream serialization, so that it may start while the
+// preceding grid on the stream finishes: W is read before that grid has completed (it
+// must not be written by it), X only after. Its own successor may start early likewise.
 cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t ldx, int rows, int ntok, int kdim,
-                             void* out, int64_t ldo, float* part, cudaStream_t stream);
+                             void* out, int64_t ldo, float* part, cudaStream_t stream, bool pdl = false);
 constexpr int SWAP_MAX_TOKENS = 256;
 
 // Whether the CTA-pair kernels are enabled (ESPACE_DISABLE_PAIR_GEMM=1 turns them off).

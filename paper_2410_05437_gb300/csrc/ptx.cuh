@@ -133,6 +133,19 @@ __device__ __forceinline__ uint64_t cleanup_limit(uint64_t limit_ns)
     return limit_ns > CLEANUP_WAIT_NS ? limit_ns : CLEANUP_WAIT_NS;
 }
 
+// ------------------------------------------------------------------------------ grid dependency
+
+// Lets the grid launched after this one on the stream (with programmatic stream
+// serialization) start once every CTA of this grid has issued this or exited.
+__device__ __forceinline__ void grid_dep_launch_dependents()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Waits until the grids this one depends on have completed and their memory operations
+// are visible (returns at once when the grid was not launched early).
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ------------------------------------------------------------------------------ TMA
 
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map)

@@ -59,6 +59,10 @@ struct TcGemmArgs {
     // the tile's other rows keep stale shared memory, which reaches only output columns past
     // `cols` (never stored) -- cheaper than the copy engine's zero fill of absent rows
     int b_rows;
+    // K-major only, launched with programmatic stream serialization: A (weights the caller
+    // guarantees the preceding grid does not write) is loaded for the first STAGES k-blocks
+    // before waiting for the preceding grid; B (tokens, maybe its output) only after
+    int pdl;
     int* status;
     uint64_t wait_limit_ns;
 };
@@ -145,16 +149,31 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int num_items = args.num_tiles * args.ksplit;
     const uint64_t limit = args.wait_limit_ns;
 
+    if (args.pdl && threadIdx.x == 0) grid_dep_launch_dependents();
+
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
+            // B loads held back until the preceding grid has completed (pdl)
+            bool dep_done = MN_MAJOR || !args.pdl;
+            int ndef = 0;
+            int def_stage[STAGES], def_kb[STAGES], def_tn[STAGES];
+            auto release_deferred = [&]() {
+                grid_dep_wait();
+                for (int q = 0; q < ndef; ++q)
+                    tma_load_2d(smem + def_stage[q] * Cfg::STAGE_BYTES + Cfg::A_BYTES, &map_b, &full[def_stage[q]],
+                                def_kb[q] * BK, def_tn[q] * BN);
+                ndef = 0;
+                dep_done = true;
+            };
             for (int item = blockIdx.x; ok && item < num_items; item += gridDim.x) {
                 int tm, tn, kb0, kb1;
                 decode_item(args, item, tm, tn, kb0, kb1);
                 for (int kb = kb0; kb < kb1; ++kb) {
+                    if (!dep_done && ndef == STAGES) release_deferred();
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
                         ok = false;
@@ -175,7 +194,14 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                                         kb * BK);
                     } else {
                         tma_load_2d(sa, &map_a, &full[stage], kb * BK, tm * BM);
-                        tma_load_2d(sb, &map_b, &full[stage], kb * BK, tn * BN);
+                        if (dep_done) {
+                            tma_load_2d(sb, &map_b, &full[stage], kb * BK, tn * BN);
+                        } else {
+                            def_stage[ndef] = stage;
+                            def_kb[ndef] = kb;
+                            def_tn[ndef] = tn;
+                            ++ndef;
+                        }
                     }
                     if (++stage == STAGES) {
                         stage = 0;
@@ -183,6 +209,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                     }
                 }
             }
+            if (!dep_done) release_deferred();   // also after giving up: the stages expect B
             if (!ok) settle_copies();
         }
     } else if (warp == 1) {
@@ -1091,6 +1118,20 @@ cudaError_t launch_kernel(const CUtensorMap& ma, const CUtensorMap& mb, const Tc
         if (e != cudaSuccess) return e;
         attr_set[device].store(true, std::memory_order_release);
     }
+    if (args.pdl) {
+        // may start while the preceding grid on the stream finishes (see TcGemmArgs::pdl)
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(grid);
+        cfg.blockDim = dim3(GEMM_THREADS);
+        cfg.dynamicSmemBytes = Cfg::SMEM_BYTES;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, kern, ma, mb, args);
+    }
     kern<<<grid, GEMM_THREADS, Cfg::SMEM_BYTES, stream>>>(ma, mb, args);
     return cudaGetLastError();
 }
@@ -1268,9 +1309,15 @@ SwapPlan gemm_swap_plan(int rows, int ntok, int kdim, int num_sms, bool allow_sp
 // tokens and the bf16 results written along rows, both coalesced, through shared memory.
 __global__ void __launch_bounds__(1024) reduce_splits_kernel(const float* __restrict__ part, int ksplit, int rows,
                                                              int64_t ld_part, int ntok, __nv_bfloat16* __restrict__ out,
-                                                             int64_t ldo)
+                                                             int64_t ldo, int pdl)
 {
     __shared__ float tile[32][33];
+    if (pdl) {
+        // launched early: let the next grid start its own weight loads, then wait for the
+        // partials of the preceding one
+        if (threadIdx.x == 0) grid_dep_launch_dependents();
+        grid_dep_wait();
+    }
     const int r0 = blockIdx.x * 32, n0 = blockIdx.y * 32;
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     float acc = 0.f;
@@ -1296,7 +1343,7 @@ __global__ void __launch_bounds__(1024) reduce_splits_kernel(const float* __rest
 }
 
 cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t ldx, int rows, int ntok, int kdim,
-                             void* out, int64_t ldo, float* part, cudaStream_t stream)
+                             void* out, int64_t ldo, float* part, cudaStream_t stream, bool pdl)
 {
     if (rows <= 0 || ntok <= 0) return cudaSuccess;
     DeviceInfo* dev = nullptr;
@@ -1322,6 +1369,7 @@ cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t 
     a.part = part;
     a.ld_part = pl.ld_part;
     a.b_rows = b_rows;
+    a.pdl = pdl ? 1 : 0;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
     const int grid = std::min(pl.tiles * pl.ksplit, dev->num_sms);
@@ -1330,8 +1378,22 @@ cudaError_t launch_gemm_swap(const void* W, int64_t ldw, const void* X, int64_t 
                                      : launch_kernel<256, 4, false, EPI_SPLIT_BF16_T>(ma, mb, a, grid, stream);
         if (e != cudaSuccess) return e;
         const dim3 grid_r((rows + 31) / 32, (ntok + 31) / 32);
+        if (pdl) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = grid_r;
+            cfg.blockDim = dim3(1024);
+            cfg.dynamicSmemBytes = 0;
+            cfg.stream = stream;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+            attr[0].val.programmaticStreamSerializationAllowed = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            return cudaLaunchKernelEx(&cfg, reduce_splits_kernel, static_cast<const float*>(part), pl.ksplit, rows,
+                                      pl.ld_part, ntok, static_cast<__nv_bfloat16*>(out), ldo, 1);
+        }
         reduce_splits_kernel<<<grid_r, 1024, 0, stream>>>(part, pl.ksplit, rows, pl.ld_part, ntok,
-                                                         static_cast<__nv_bfloat16*>(out), ldo);
+                                                         static_cast<__nv_bfloat16*>(out), ldo, 0);
         return cudaGetLastError();
     }
     if (pl.bn == 128) return launch_kernel<128, 6, false, EPI_STORE_BF16_T>(ma, mb, a, grid, stream);

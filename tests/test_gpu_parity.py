@@ -973,3 +973,112 @@ def test_forward_after_a_launch_that_gave_up(esp, N):
             assert_y_close(Y, Y_o)
     finally:
         esp.espace_proj_destroy(p)
+
+
+# ------------------------------------------------------------------------------ degenerate calibrations
+
+def test_build_projection_rank_deficient_calibration(esp):
+    """Fewer calibration tokens (64) than features (256): C has rank 64, so with L = 128 the
+    projection keeps all of the calibration variance (Thm. 1: the discarded eigenvalues are
+    zero) and its extra columns span part of C's null space, where any orthonormal choice is
+    right. Checked: eigenvalues against the oracle (zero beyond the rank, within the fp32
+    sums), orthonormal P within bf16 rounding, the MSE of Eq. 6 on the calibration tokens
+    near zero, and the forward with the library's P."""
+    K, M, L, n, N = 256, 192, 128, 64, 100
+    model = synth.ActivationModel(K, seed=31)
+    Xc = model.sample(n, stream="calib_tokens")
+    X = model.sample(N)
+    W = synth.weights(M, K, seed=31)
+    h = esp.espace_calib_create(K)
+    p = None
+    try:
+        esp.espace_calib_accumulate(h, dev(Xc))
+        p = esp.espace_build_projection(h, dev(W), L)
+        w = esp.espace_proj_eigenvalues(p)
+        Pb = synth.bf16_to_f64(torch.from_numpy(esp.espace_proj_read_P(p).view(np.int16)).view(torch.bfloat16))
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Y)
+        torch.cuda.synchronize()
+        esp.espace_check()
+    finally:
+        if p:
+            esp.espace_proj_destroy(p)
+        esp.espace_calib_destroy(h)
+    w_o = oracle.eigh(oracle.autocorr_sum(f64(Xc)) / n)[0]
+    assert np.allclose(w, w_o, rtol=0, atol=1e-5 * w_o[0])
+    assert np.all(np.abs(w[n:]) <= 1e-5 * w_o[0])
+    assert np.abs(Pb.T @ Pb - np.eye(L)).max() < 2e-2
+    mse = oracle.projection_mse(f64(Xc), Pb)
+    total = oracle.projection_mse(f64(Xc), np.zeros((K, 1)))          # E ||x||^2
+    assert mse <= 1e-4 * total, (mse, total)
+    assert_y_close(Y, oracle.forward(f64(X), Pb, f64(W))[0])
+
+
+def test_build_projection_from_all_zero_calibration(esp):
+    """All-zero calibration tokens: C = 0, every eigenvalue is zero and every orthonormal P
+    is optimal (Thm. 1). The build must still give orthonormal columns (bf16) and a working
+    layer: the forward matches the oracle fed the library's P."""
+    K, M, L, n, N = 64, 96, 16, 100, 40
+    h = esp.espace_calib_create(K)
+    p = None
+    try:
+        esp.espace_calib_accumulate(h, torch.zeros((n, K), dtype=torch.bfloat16, device="cuda"))
+        p = esp.espace_build_projection(h, dev(synth.weights(M, K, seed=32)), L)
+        w = esp.espace_proj_eigenvalues(p)
+        Pb = synth.bf16_to_f64(torch.from_numpy(esp.espace_proj_read_P(p).view(np.int16)).view(torch.bfloat16))
+        X = synth.ActivationModel(K, seed=32).sample(N)
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, dev(X), Y)
+        torch.cuda.synchronize()
+        esp.espace_check()
+    finally:
+        if p:
+            esp.espace_proj_destroy(p)
+        esp.espace_calib_destroy(h)
+    assert np.all(w == 0)
+    assert np.abs(Pb.T @ Pb - np.eye(L)).max() < 2e-2
+    assert_y_close(Y, oracle.forward(f64(X), Pb, f64(synth.weights(M, K, seed=32)))[0])
+
+
+@pytest.mark.parametrize("N", [24, 64, 200])
+def test_few_token_chain_reads_each_input_after_it_is_written(esp, N):
+    """A chain of few-token layers on one stream with no synchronization between them: each
+    layer's input is the previous one's output (buffers filled with NaN first), projected and
+    dense layers interleaved. The few-token launches may start while the previous kernel
+    finishes and load their weights early, but must read their tokens only after it has
+    completed: every output must equal the oracle applied to the input it was given."""
+    K = M = 1024
+    L = 512
+    torch.cuda.synchronize()
+    Ws = [synth.weights(M, K, seed=90 + i) for i in range(4)]
+    ps = [esp.espace_proj_from_host(synth.random_projection(K, L, seed=90 + i), dev(Ws[i])) for i in range(3)]
+    try:
+        X0 = dev(synth.ActivationModel(K, seed=90).sample(N))
+        W3 = dev(Ws[3])
+        outs = [torch.full((N, M), float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(6)]
+        torch.cuda.synchronize()
+        x = X0
+        kinds = []
+        for i, y in enumerate(outs):
+            if i % 2 == 1:
+                esp.espace_dense_forward(x, W3, y)
+                kinds.append("dense")
+            else:
+                esp.espace_linear_forward(ps[i // 2], x, y)
+                kinds.append(i // 2)
+            x = y
+        torch.cuda.synchronize()
+        esp.espace_check()
+        x = X0
+        for kind, y in zip(kinds, outs):
+            xf = f64(x)
+            if kind == "dense":
+                ref = oracle.dense(xf, f64(Ws[3]))
+            else:
+                Pb = oracle.bf16_round(synth.random_projection(K, L, seed=90 + kind))
+                ref = oracle.forward(xf, Pb, f64(Ws[kind]))[0]
+            assert_y_close(y, ref)
+            x = y
+    finally:
+        for p in ps:
+            esp.espace_proj_destroy(p)
