@@ -275,9 +275,10 @@ int espace_proj_tp_info(espace_proj_t p, int* kind, int* tp);
  * (one more launch adds the fp32 partials in a fixed order, so results are reproducible bit
  * for bit); larger N runs one persistent tcgen05 launch holding both products, except that
  * a layer with K >= 2 M whose Z has fewer 256 x 256 tiles than a quarter of the SMs runs
- * phase 1 as a split product and phase 2 on CTA pairs. The few-token launches (N <= 256)
- * may start streaming the handle's P and W' while the kernel before them on the stream
- * finishes (programmatic dependent launch); they read X_dev only after it has completed.
+ * phase 1 as a split product and phase 2 on CTA pairs. The few-token and decode launches
+ * (N <= 256) may start streaming the handle's P and W' while the kernel before them on the
+ * stream finishes (programmatic dependent launch); they read X_dev only after it has
+ * completed.
  * N = 0 is a no-op. The first call
  * with a larger N than any before on this handle allocates the Z scratch and the split
  * workspace (synchronously, so outside a stream capture); later calls allocate nothing. */
@@ -352,7 +353,7 @@ int espace_linear_forward_noalloc(espace_proj_t p, const void* X_dev, int64_t N,
  * the first such call allocates, or grows, and so must make outside a stream capture;
  * above: tcgen05): the baseline the projected layer is measured against. Calls that split
  * share the device's workspace: order them on the GPU (one stream, or streams that wait on
- * each other). For 9 <= N <= 256 the product may start reading W_dev while the kernel
+ * each other). For N <= 256 the product may start reading W_dev while the kernel
  * launched just before it on the stream finishes, when that kernel is one of this
  * library's few-token products (programmatic dependent launch); X_dev is read only after
  * that kernel completes. So W_dev must not be written by the call made just before on

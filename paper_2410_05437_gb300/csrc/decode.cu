@@ -74,6 +74,10 @@ struct DecodeArgs {
     int tok_elems;               // one token (N = 1): bf16 values of its shared-memory copy
     int slot_floats;             // 16-warp groups: floats of the partial-sum slots
     unsigned int* bar;           // grid barrier counter
+    // launched with programmatic stream serialization: the producer streams the weights
+    // (which the preceding grid must not write) before that grid has completed; the
+    // consumers wait for it before reading tokens or touching the barrier counter
+    int pdl;
     int* status;
     uint64_t wait_limit_ns;
     // CTA b owns rows [cut[p][b], cut[p][b + 1]) of phase p (computed on the host)
@@ -375,6 +379,7 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
     for (int i = threadIdx.x; i < a.acc_rows * C::NTP; i += blockDim.x) acc[i] = 0.f;
     __syncthreads();
     volatile int* abort = &abort_s;
+    if (a.pdl && threadIdx.x == 0) grid_dep_launch_dependents();
 
     if (warp == DEC_CWARPS) {
         // ------------------------------------------------------------ producer (one thread)
@@ -425,6 +430,8 @@ __global__ void __launch_bounds__(DEC_THREADS, 1) decode_kernel(const DecodeArgs
 
     // ---------------------------------------------------------------- consumers (16 warps)
     const int group = warp / C::WPS, u = warp % C::WPS;
+    // tokens, Z and the barrier counter may belong to the preceding grid until it completes
+    if (a.pdl) grid_dep_wait();
     // the grid barrier's bit before this CTA arrives (it cannot flip earlier)
     const unsigned bar_start = (a.phases > 1 && threadIdx.x == 0) ? ld_acquire_gpu(a.bar) : 0u;
     int j0 = 0;   // ring index of the phase's first stage
@@ -611,14 +618,28 @@ cudaError_t launch_t(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev,
     a.tok_elems = pl.tok_elems;
     a.slot_floats = pl.slot_floats;
     std::copy(&pl.cut[0][0], &pl.cut[0][0] + 2 * (DEC_MAX_GRID + 1), &a.cut[0][0]);
-    if (a.phases == 1) {
-        // no grid barrier: an ordinary launch
-        kern<<<dev->num_sms, DEC_THREADS, pl.smem, stream>>>(a);
-        return cudaGetLastError();
+    // programmatic stream serialization (see DecodeArgs::pdl), with a cooperative launch for
+    // the grid barrier of the two-phase form
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(dev->num_sms);
+    cfg.blockDim = dim3(DEC_THREADS);
+    cfg.dynamicSmemBytes = static_cast<size_t>(pl.smem);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[2];
+    int na = 0;
+    if (a.pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
     }
-    void* params[] = {&a};
-    return cudaLaunchCooperativeKernel(reinterpret_cast<void*>(kern), dim3(dev->num_sms), dim3(DEC_THREADS),
-                                       params, static_cast<size_t>(pl.smem), stream);
+    if (a.phases > 1) {
+        attr[na].id = cudaLaunchAttributeCooperative;
+        attr[na].val.cooperative = 1;
+        ++na;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = na;
+    return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
 cudaError_t launch_any(DecodeArgs& a, const DecodePlan& pl, const DeviceInfo* dev, cudaStream_t stream)
@@ -667,6 +688,7 @@ cudaError_t launch_decode_forward(const void* PT, const void* WfT, const void* X
     a.phases = 2;
     a.nt = nt;
     a.bar = grid_bar;
+    a.pdl = 1;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
     return launch_any(a, pl, dev, stream);
@@ -689,6 +711,7 @@ cudaError_t launch_decode_dense(const void* W, const void* X, void* Y, int K, in
     a.phases = 1;
     a.nt = nt;
     a.bar = nullptr;
+    a.pdl = 1;
     a.status = dev->status;
     a.wait_limit_ns = wait_limit_ns();
     return launch_any(a, pl, dev, stream);
