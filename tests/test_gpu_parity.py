@@ -158,6 +158,9 @@ FORWARD_CASES = [
     (1, 24, 8, 1, 0),              # rank 1
     (1, 16384, 264, 128, 0),       # large K, few output rows
     (1, 24576, 512, 128, 2),       # K of the GPT3-22B FC2 layer
+    # phase 2 over several 2048-wide k-blocks of Z, the last one ragged
+    (4, 8192, 520, 4500, 2),       # three k-blocks, ragged M tail
+    (32, 4096, 776, 3000, 2),      # two k-blocks, 32-token groups
 ]
 
 
@@ -936,13 +939,14 @@ def test_fused_forward_completes_while_other_work_holds_half_the_sms(esp):
         esp.espace_proj_destroy(p)
 
 
-@pytest.mark.parametrize("N", [2048, 4])
-def test_forward_after_a_launch_that_gave_up(esp, N):
+@pytest.mark.parametrize("N,K,L", [(2048, 1024, 512), (4, 1024, 512), (4, 2048, 1536)])
+def test_forward_after_a_launch_that_gave_up(esp, N, K, L):
     """A launch whose waits give up (a 2 us limit) leaves the handle's counters consistent:
     the fused kernel's last CTA zeroes its readiness counters, ticket and exit counter on
-    every exit path, and every CTA of the decode kernel arrives once at its grid barrier.
-    The timeout is reported, and the next forwards on the same handle are right."""
-    K, M, L = 1024, 2048, 512
+    every exit path, and every CTA of the decode kernel arrives once at its grid barrier
+    (whose second phase runs over one k-block of Z at L = 512, two at L = 1536). The timeout
+    is reported, and the next forwards on the same handle are right."""
+    M = 2048
     p, Xd, Y_o = _layer_and_reference(esp, K, M, L, N, seed=78)
     try:
         Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
@@ -1040,7 +1044,7 @@ def test_build_projection_from_all_zero_calibration(esp):
     assert_y_close(Y, oracle.forward(f64(X), Pb, f64(synth.weights(M, K, seed=32)))[0])
 
 
-@pytest.mark.parametrize("N", [24, 64, 200])
+@pytest.mark.parametrize("N", [4, 24, 64, 200])
 def test_few_token_chain_reads_each_input_after_it_is_written(esp, N):
     """A chain of few-token layers on one stream with no synchronization between them: each
     layer's input is the previous one's output (buffers filled with NaN first), projected and
