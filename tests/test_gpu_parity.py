@@ -939,6 +939,46 @@ def test_fused_forward_completes_while_other_work_holds_half_the_sms(esp):
         esp.espace_proj_destroy(p)
 
 
+@pytest.mark.parametrize("N", [1, 8, 24])
+def test_decode_forward_completes_while_other_work_holds_half_the_sms(esp, N):
+    """The decode kernel's two products meet at a grid barrier, so it is a cooperative
+    launch: with half of the SMs held by another stream's kernel (300 ms), it starts once all
+    of its CTAs can be resident, and none of its bounded waits counts the time before that.
+    Within a 50 ms wait limit it completes with the right result, and so does the next call
+    on the handle (24 tokens: the decode kernel forced, two token tiles)."""
+    K, M, L = 2048, 2048, 1024
+    p, Xd, Y_o = _layer_and_reference(esp, K, M, L, N, seed=79)
+    try:
+        path = esp.PATH_SMALL_N if N > 16 else esp.PATH_AUTO
+        assert esp.espace_linear_forward_launches(p, N, path) == 1
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward_path(p, Xd, Y, path)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        assert_y_close(Y, Y_o)
+        Y.fill_(float("nan"))
+        sms = torch.cuda.get_device_properties(0).multi_processor_count
+        side = torch.cuda.Stream()
+        torch.cuda.synchronize()
+        esp.espace_set_wait_limit_ns(50_000_000)
+        try:
+            esp.espace_debug_occupy(sms // 2, 300_000_000, side)
+            time.sleep(0.02)                            # the holding CTAs are resident
+            esp.espace_linear_forward_path(p, Xd, Y, path)
+            torch.cuda.synchronize()
+        finally:
+            esp.espace_set_wait_limit_ns(4_000_000_000)
+        esp.espace_check()                              # no wait gave up
+        assert_y_close(Y, Y_o)
+        Y.fill_(float("nan"))
+        esp.espace_linear_forward_path(p, Xd, Y, path)  # and the next call on the handle
+        torch.cuda.synchronize()
+        esp.espace_check()
+        assert_y_close(Y, Y_o)
+    finally:
+        esp.espace_proj_destroy(p)
+
+
 @pytest.mark.parametrize("N,K,L", [(2048, 1024, 512), (4, 1024, 512), (4, 2048, 1536)])
 def test_forward_after_a_launch_that_gave_up(esp, N, K, L):
     """A launch whose waits give up (a 2 us limit) leaves the handle's counters consistent:
