@@ -1463,12 +1463,13 @@ int2* syrk_tiles(int K, int tile_rows, int tile_cols, int* count)
 }
 
 // Token splits per tile: the count s that minimises the last worker's time, ceil(tiles s /
-// workers) waves of ceil(kblocks / s) k-blocks plus a per-item epilogue (the atomic adds of
-// a 256 x 256 fp32 tile, taken as 8 k-blocks of MMA), with at least 16 k-blocks (1024
-// tokens) per split; more splits are taken only for a modelled gain of 2% or more.
-void choose_splits(int kblocks, int tiles, int workers, int* ksplit, int* kb_per_split)
+// workers) waves of ceil(kblocks / s) k-blocks plus a per-item cost of item_kb k-blocks of
+// MMA (the atomic adds of a 256 x 256 fp32 tile and the item's pipeline fill), with at least
+// 16 k-blocks (1024 tokens) per split; more splits are taken only for a modelled gain of 2%
+// or more. The per-item cost is the caller's, measured for its kind of launch.
+void choose_splits(int kblocks, int tiles, int workers, int64_t item_kb, int* ksplit, int* kb_per_split)
 {
-    constexpr int64_t EPILOGUE_KB = 8;
+    const int64_t EPILOGUE_KB = item_kb;
     int best_s = 1;
     int64_t best = INT64_MAX;
     for (int s = 1; s <= 64; ++s) {
@@ -1505,7 +1506,7 @@ cudaError_t launch_syrk_upper_two(const void* X, const void* Y, int64_t N, int K
     if (pair) {
         int count = 0;
         if (syrk_tiles(K, PAIR_BM, PAIR_BN, &count) == nullptr) return cudaErrorMemoryAllocation;
-        choose_splits(kblocks, 2 * count, dev->num_sms / 2, &ksplit, &kbps);
+        choose_splits(kblocks, 2 * count, dev->num_sms / 2, 8, &ksplit, &kbps);
     }
     if (assign && (!pair || ksplit > 1)) {
         // split reductions add: start from zero
@@ -1582,7 +1583,9 @@ cudaError_t launch_syrk_segments_upper(const void* Q, int64_t q_rows, int K, int
     p.kblocks = nseg * (seg_rows / BK);
     p.tiles_n = 0;
     p.num_tiles = count;
-    choose_splits(p.kblocks, count, dev->num_sms / 2, &p.ksplit, &p.kb_per_split);
+    // (8 k-blocks per item: five splits of the NL-MSE products at K = 4096 measured 498 us a
+    // call, one split 512 us)
+    choose_splits(p.kblocks, count, dev->num_sms / 2, 8, &p.ksplit, &p.kb_per_split);
     p.tile_list = tiles;
     p.out = S;
     p.ldo = K;
@@ -1621,7 +1624,9 @@ cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int
         p.kblocks = kblocks;
         p.tiles_n = 0;
         p.num_tiles = count;
-        choose_splits(kblocks, count, dev->num_sms / 2, &p.ksplit, &p.kb_per_split);
+        // (24 k-blocks per item: at K = 4096 over 65,536 tokens one split measured 0.670 ms,
+        // the five that 8 k-blocks per item pick 0.685 ms; K = 6144 and 24576 take one either way)
+        choose_splits(kblocks, count, dev->num_sms / 2, 24, &p.ksplit, &p.kb_per_split);
         p.tile_list = tiles;
         p.out = S;
         p.ldo = K;
@@ -1675,7 +1680,7 @@ cudaError_t launch_gemm_tn_tokens_f32(const void* U, int R, const void* V, int C
     p.kblocks = static_cast<int>((N + BK - 1) / BK);
     p.tiles_n = (C + PAIR_BN - 1) / PAIR_BN;
     p.num_tiles = ((R + PAIR_BM - 1) / PAIR_BM) * p.tiles_n;
-    choose_splits(p.kblocks, p.num_tiles, dev->num_sms / 2, &p.ksplit, &p.kb_per_split);
+    choose_splits(p.kblocks, p.num_tiles, dev->num_sms / 2, 8, &p.ksplit, &p.kb_per_split);
     p.tile_list = nullptr;
     p.out = out;
     p.ldo = ldo;
