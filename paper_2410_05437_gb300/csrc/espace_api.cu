@@ -198,6 +198,7 @@ struct espace_calib_s {
     int64_t K = 0;
     int device = 0;
     float* S = nullptr;            // [K][K] fp32, upper triangle valid
+    int* sched = nullptr;          // the SYRK's wave and exit counters (zeroed; left zero)
     int64_t n = 0;
     int mode = 0;                  // 0 unset, 1 plain, 2 normalized (Cor. 1), 3 NL-MSE (Thm. 2),
                                    // 4 NL-MSE with L2-normalized tokens and gradients
@@ -302,10 +303,13 @@ int espace_calib_create(int64_t K, espace_calib_t* out)
                     (long long)(sizeof(float) * K * K), cudaGetErrorString(e));
     }
     e = cudaMemset(h->S, 0, sizeof(float) * K * K);
+    if (e == cudaSuccess) e = cudaMalloc(&h->sched, 64);
+    if (e == cudaSuccess) e = cudaMemset(h->sched, 0, 64);
     if (e != cudaSuccess) {
         cudaFree(h->S);
+        if (h->sched) cudaFree(h->sched);
         delete h;
-        return fail_cuda(e, "espace_calib_create: cudaMemset");
+        return fail_cuda(e, "espace_calib_create: scratch");
     }
     *out = h;
     return ESPACE_OK;
@@ -338,7 +342,7 @@ static int calib_accumulate_impl(espace_calib_t h, const void* X, int64_t N, voi
         CUDA_TRY(launch_normalize_rows(X, N, static_cast<int>(h->K), h->xn, st), "normalize_rows launch");
         src = h->xn;
     }
-    CUDA_TRY(launch_syrk_upper(src, N, static_cast<int>(h->K), h->S, st), "syrk launch");
+    CUDA_TRY(launch_syrk_upper(src, N, static_cast<int>(h->K), h->S, st, h->sched), "syrk launch");
     h->mode = mode;
     h->n += N;
     return ESPACE_OK;
@@ -506,6 +510,7 @@ void espace_calib_destroy(espace_calib_t h)
     DeviceGuard g(h->device);
     cudaDeviceSynchronize();
     if (h->S) cudaFree(h->S);
+    if (h->sched) cudaFree(h->sched);
     if (h->xn) cudaFree(h->xn);
     if (h->nl_f32) cudaFree(h->nl_f32);
     if (h->nl_bf) cudaFree(h->nl_bf);

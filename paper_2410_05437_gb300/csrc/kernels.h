@@ -83,13 +83,17 @@ cudaError_t launch_gemm_tn_tokens_f32(const void* U, int R, const void* V, int C
 cudaError_t launch_syrk_segments_upper(const void* Q, int64_t q_rows, int K, int seg_rows, int nseg,
                                        const int* seg_u, const int* seg_v, float* S, cudaStream_t stream);
 // S[K][K] (fp32, upper triangle i <= j) += X^T X for X[N][K] bf16, on tcgen05 tensor cores.
-cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream);
+// sched: two ints of the caller, zero before the first launch and left zero by every launch
+// (the pair kernel's wave counter and exit counter; nullptr: no wave pacing).
+cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream,
+                              int* sched = nullptr);
 // Two independent SYRKs in one launch: Sx += X^T X and Sy += Y^T Y (upper triangles), or
 // Sx = X^T X and Sy = Y^T Y with assign (the lower triangles are then left unset).
 cudaError_t launch_syrk_upper_two(const void* X, const void* Y, int64_t N, int K, float* Sx, float* Sy,
                                   bool assign, cudaStream_t stream);
 // The same kernel with two operands: S's upper triangle += that of X^T Y (X, Y [N][K] bf16).
-cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream);
+cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream,
+                                    int* sched = nullptr);
 
 // Token counts served by the decode kernels (when asked for), and chosen for them by the
 // automatic paths: above these, the swapped tcgen05 products measured faster.

@@ -380,6 +380,8 @@ constexpr int PAIR_EPI_BYTES = 4 * 2 * PAIR_EPI_BUF;
 // tokens) and its epilogue adds the chunks in fp32 registers, so that long token runs do
 // not lose precision in the tensor core's accumulator.
 constexpr int SYRK_CHUNK = 16;
+// Longest wait of a pair for the previous wave of items (PairArgs::wave_ctr).
+constexpr uint64_t WAVE_WAIT_NS = 20000;
 // Tile rows per group of the grouped tile order of full-grid products.
 constexpr int PAIR_GROUP_M = 8;
 // Diagonal blocks of a block-diagonal product (one per tensor-parallel rank).
@@ -439,7 +441,13 @@ struct PairArgs {
     int* ready;
     int nready;
     int* ticket;      // work-item ticket, or nullptr for the static order
-    int* exit_ctr;    // CTAs that left (with a ticket)
+    int* exit_ctr;    // CTAs that left (with a ticket or a wave counter)
+    // token-reduction programs over many waves of items (static order): items whose loads
+    // both CTAs of their pair have issued. A pair starts its i-th item once every pair has
+    // issued the loads of its (i-1)-th, so that the pairs of a wave stream the same token
+    // rows of the feature slices they share, and those rows are read from L2; the wait is
+    // only a hint (at most WAVE_WAIT_NS), and nothing depends on it for correctness
+    int* wave_ctr;
     int* status;
     uint64_t wait_limit_ns;
     int nblocks;
@@ -735,6 +743,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                 pair_block_of(args, prob, tn, 0, ak0, brow, ccol, cend);
                 const int row_a = tm * PAIR_BM + static_cast<int>(rank) * 128;
                 const int row_b = brow + static_cast<int>(rank) * 128;
+                if (SYRK && args.wave_ctr != nullptr) {
+                    // this pair's i-th item is in wave i (static order): wait, a bounded
+                    // while, for both CTAs of every pair to have issued their wave i - 1
+                    const int target = 2 * npairs * i;
+                    const uint64_t g0 = globaltimer_ns();
+                    while (*reinterpret_cast<volatile int*>(args.wave_ctr) < target &&
+                           globaltimer_ns() - g0 < WAVE_WAIT_NS)
+                        __nanosleep(256);
+                }
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.status, limit,
                                    ESPACE_ERR_TIMEOUT)) {
@@ -765,6 +782,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
                         phase ^= 1u;
                     }
                 }
+                if (SYRK && args.wave_ctr != nullptr) atomicAdd(args.wave_ctr, 1);
             }
             if (!ok) settle_copies();
         }
@@ -1053,7 +1071,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairShape<SYRK>::THR
             __threadfence();
             volatile int* r = args.ready;
             for (int b = 0; b < args.nready; ++b) r[b] = 0;
-            *reinterpret_cast<volatile int*>(args.ticket) = 0;
+            if (args.ticket != nullptr) *reinterpret_cast<volatile int*>(args.ticket) = 0;
+            if (args.wave_ctr != nullptr) *reinterpret_cast<volatile int*>(args.wave_ctr) = 0;
             __threadfence();
             *reinterpret_cast<volatile int*>(args.exit_ctr) = 0;
         }
@@ -1489,9 +1508,9 @@ void choose_splits(int kblocks, int tiles, int workers, int64_t item_kb, int* ks
 
 }  // namespace
 
-cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream)
+cudaError_t launch_syrk_upper(const void* X, int64_t N, int K, float* S, cudaStream_t stream, int* sched)
 {
-    return launch_syrk_cross_upper(X, X, N, K, S, stream);
+    return launch_syrk_cross_upper(X, X, N, K, S, stream, sched);
 }
 
 cudaError_t launch_syrk_upper_two(const void* X, const void* Y, int64_t N, int K, float* Sx, float* Sy,
@@ -1601,7 +1620,8 @@ cudaError_t launch_syrk_segments_upper(const void* Q, int64_t q_rows, int K, int
     return launch_pair<true>(maps, a, dev, stream);
 }
 
-cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream)
+cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int K, float* S, cudaStream_t stream,
+                                    int* sched)
 {
     if (N <= 0) return cudaSuccess;
     DeviceInfo* dev = nullptr;
@@ -1632,6 +1652,13 @@ cudaError_t launch_syrk_cross_upper(const void* X, const void* Y, int64_t N, int
         p.ldo = K;
         p.upper = 1;
         a.nprob = 1;
+        // many waves of items (K = 24576: 4656 tiles, 62 waves): keep the pairs' waves
+        // together (PairArgs::wave_ctr; measured 28.1-28.3 -> 25.1-27.5 ms for 65,536 tokens).
+        // With 2-4 waves (K <= 6144) the pairs hardly drift apart and the waits cost about 1%.
+        if (sched != nullptr && static_cast<int64_t>(count) * p.ksplit >= 16LL * (dev->num_sms / 2)) {
+            a.wave_ctr = sched;
+            a.exit_ctr = sched + 1;
+        }
         a.status = dev->status;
         a.wait_limit_ns = wait_limit_ns();
         return launch_pair<true>(maps, a, dev, stream);

@@ -135,6 +135,35 @@ def test_gpt3_22b_calibration_rows(esp, K):
         esp.espace_calib_destroy(h)
 
 
+def test_calibration_1m_tokens_chunking_invariance(esp):
+    """The 1,048,576-token calibration at K = 6144 (the GPT3-22B QKV / FC1 input) is timed,
+    not compared with the fp64 oracle (a 1M x 6144 reduction in fp64 on the host takes far
+    too long); instead S over the same tokens fed as 16 chunks of 65,536 and as 64 chunks of
+    16,384 agree to fp32 summation-order error, with the same count (Eq. 4's sum does not
+    depend on how the tokens are batched). Each call adds its 1024-token TMEM sums into S in
+    fp32, so an entry takes 16 or 64 more fp32 roundings: at most 64 * 2^-24 = 3.8e-6
+    relative between the two."""
+    K, total = 6144, 1 << 20
+    model = synth.ActivationModel(K, seed=synth.config_seed("gpt3_22b_qkv"))
+    S = []
+    for chunk in (65536, 16384):
+        h = esp.espace_calib_create(K)
+        try:
+            for c in range(total // 65536):
+                Xd = model.sample_device(65536, stream="calib_tokens", chunk=c)
+                for off in range(0, 65536, chunk):
+                    esp.espace_calib_accumulate(h, Xd[off:off + chunk])
+                del Xd
+            Sh, cnt = esp.espace_calib_export(h, K)
+            esp.espace_check()
+            assert cnt == total
+            S.append(np.triu(Sh))
+        finally:
+            esp.espace_calib_destroy(h)
+    err = np.linalg.norm(S[0] - S[1]) / np.linalg.norm(S[1])
+    assert err <= 64 * 2.0 ** -24, f"chunkings differ by {err:.3e} normwise"
+
+
 # ------------------------------------------------------------------ decode-shaped token sweep
 
 @pytest.mark.parametrize("layer", ["qkv", "o", "gate_up", "down"])
