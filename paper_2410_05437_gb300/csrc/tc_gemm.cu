@@ -1488,7 +1488,6 @@ int2* syrk_tiles(int K, int tile_rows, int tile_cols, int* count)
 // or more. The per-item cost is the caller's, measured for its kind of launch.
 void choose_splits(int kblocks, int tiles, int workers, int64_t item_kb, int* ksplit, int* kb_per_split)
 {
-    const int64_t EPILOGUE_KB = item_kb;
     int best_s = 1;
     int64_t best = INT64_MAX;
     for (int s = 1; s <= 64; ++s) {
@@ -1496,7 +1495,7 @@ void choose_splits(int kblocks, int tiles, int workers, int64_t item_kb, int* ks
         if (s > 1 && kbps < 16) break;
         if ((kblocks + kbps - 1) / kbps != s) continue;   // the same split as a smaller s
         const int64_t waves = (static_cast<int64_t>(tiles) * s + workers - 1) / workers;
-        const int64_t cost = waves * (kbps + EPILOGUE_KB);
+        const int64_t cost = waves * (kbps + item_kb);
         if (cost * 50 < best * 49) {
             best = cost;
             best_s = s;
