@@ -317,6 +317,18 @@ int espace_linear_forward_launches(espace_proj_t p, int64_t N, int path);
 int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host,
                                void* stream);
 
+/* Async. espace_linear_forward_host without the final wait: the copies and products are
+ * queued as described there, the caller's stream is ordered after the last copy out, and the
+ * call returns. X_host must not change, and Y_host is not filled, until the caller's stream
+ * reaches that point (synchronize it, or an event recorded on it after the call). Calls on
+ * one handle must be ordered on one stream (they share the handle's staging); independent
+ * layers on separate streams overlap one layer's copies with another's products. The first
+ * call with a larger N than any before synchronizes the stream and allocates the staging
+ * (outside a stream capture). An error after copies were queued waits for them before
+ * returning, so no copy touches the host buffers after an error return. */
+int espace_linear_forward_host_async(espace_proj_t p, const void* X_host, int64_t N, void* Y_host,
+                                     void* stream);
+
 /* Capacity, in bf16 values, of the fixed scratch used by espace_linear_forward_noalloc:
  * 16 MiB, enough for N * Lp <= 8,388,608 (e.g. 4096 tokens at L = 2048). */
 #define ESPACE_NOALLOC_Z_ELEMS 8388608

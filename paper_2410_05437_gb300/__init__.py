@@ -35,7 +35,7 @@ __all__ = [
     "PATH_AUTO", "PATH_TENSOR", "PATH_SMALL_N", "PATH_TENSOR_SPLIT", "EXPORTED_SYMBOLS",
     "TP_COLUMN", "TP_ROW", "espace_proj_tp_from_host", "espace_build_projection_tp", "espace_proj_tp_info",
     "espace_calib_accumulate_nl", "espace_proj_refold", "espace_train_forward", "espace_train_backward",
-    "espace_train_weight_grad", "espace_linear_forward_host",
+    "espace_train_weight_grad", "espace_linear_forward_host", "espace_linear_forward_host_async",
     "espace_dense_backward",
     "espace_linear_forward_launches",
 ]
@@ -100,6 +100,7 @@ _SIGNATURES = {
     "espace_linear_forward_path": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp, ctypes.c_int]),
     "espace_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_linear_forward_host": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
+    "espace_linear_forward_host_async": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_linear_forward_launches": (ctypes.c_int, [_vp, _i64, ctypes.c_int]),
     "espace_dense_forward": (ctypes.c_int, [_vp, _i64, _i64, _vp, _i64, _vp, _vp]),
     "espace_proj_refold": (ctypes.c_int, [_vp, _vp, _vp]),
@@ -393,6 +394,13 @@ def espace_linear_forward_launches(p: int, N: int, path: int = PATH_AUTO) -> int
 def espace_linear_forward_host(p: int, X, Y, stream=None) -> None:
     """X [N][K] and Y [N][M]: host bf16 tensors (pinned for overlapped copies)."""
     _check(lib.espace_linear_forward_host(p, _host_ptr(X), int(X.shape[0]), _host_ptr(Y), _stream(stream)))
+
+
+def espace_linear_forward_host_async(p: int, X, Y, stream=None) -> None:
+    """As espace_linear_forward_host, returning once queued: Y is filled (and X may change)
+    only when the stream has passed this point."""
+    _check(lib.espace_linear_forward_host_async(p, _host_ptr(X), int(X.shape[0]), _host_ptr(Y),
+                                                _stream(stream)))
 
 
 def espace_linear_forward_noalloc(p: int, X, Y, N: int | None = None, stream=None) -> None:

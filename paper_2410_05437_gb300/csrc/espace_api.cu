@@ -1165,7 +1165,9 @@ static int host_chunks(int64_t N, int64_t* chunk)
     return nc;
 }
 
-int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream)
+// The host-buffer forward; wait: return only once Y_host is filled (else the caller's stream
+// is ordered after the last copy out and the call returns once everything is queued).
+static int forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream, bool wait)
 {
     if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward_host: null handle");
     if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "espace_linear_forward_host: tensor-parallel handle");
@@ -1250,12 +1252,23 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
         CUDA_TRY(cudaMemcpyAsync(yh + t0 * M, p->hy + t0 * M, sizeof(uint16_t) * n * M, cudaMemcpyDeviceToHost, p->s_out),
                  "espace_linear_forward_host: copy out");
     }
-    // the caller's stream continues after the last copy; the call returns with Y_host filled
+    // the caller's stream continues after the last copy; the synchronous form returns with
+    // Y_host filled
     CUDA_TRY(cudaEventRecord(end, p->s_out), "espace_linear_forward_host: event");
     CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host: order");
-    CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host: wait");
+    if (wait) CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host: wait");
     drain.armed = false;
     return ESPACE_OK;
+}
+
+int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream)
+{
+    return forward_host(p, X_host, N, Y_host, stream, true);
+}
+
+int espace_linear_forward_host_async(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream)
+{
+    return forward_host(p, X_host, N, Y_host, stream, false);
 }
 
 // Split workspace of the dense forward's few-token products, per device (dense calls on

@@ -253,6 +253,44 @@ def test_linear_forward_host_buffers(esp, N):
         esp.espace_proj_destroy(p)
 
 
+def test_linear_forward_host_async_two_layers_on_two_streams(esp):
+    """The asynchronous host-buffer forward: two layers, each on a stream of its own, two
+    calls each with different inputs queued back to back (the second call on a handle reuses
+    its staging, so it must run after the first), nothing waited for until both streams are
+    synchronized; every output equals the device-buffer forward bit for bit, and the oracle
+    within the tolerances."""
+    shapes = [(1024, 1000, 512, 2304), (1536, 1000, 448, 1300)]   # K < 2 M: the fused kernel
+    layers = []
+    try:
+        for i, (K, M, L, N) in enumerate(shapes):
+            model = synth.ActivationModel(K, seed=6100 + i)
+            W = synth.weights(M, K, seed=6100 + i)
+            P = synth.random_projection(K, L, seed=6100 + i)
+            p = esp.espace_proj_from_host(P, dev(W))
+            Xs = [model.sample(N, chunk=c).contiguous().pin_memory() for c in range(2)]
+            Ys = [torch.full((N, M), float("nan"), dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+            layers.append({"p": p, "P": P, "W": W, "X": Xs, "Y": Ys, "s": torch.cuda.Stream()})
+        torch.cuda.synchronize()
+        for c in range(2):
+            for l in layers:
+                esp.espace_linear_forward_host_async(l["p"], l["X"][c], l["Y"][c], l["s"])
+        for l in layers:
+            l["s"].synchronize()
+        esp.espace_check()
+        for l in layers:
+            for c in range(2):
+                N, M = l["Y"][c].shape
+                Yd = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+                esp.espace_linear_forward(l["p"], dev(l["X"][c]), Yd)
+                torch.cuda.synchronize()
+                assert torch.equal(l["Y"][c].view(torch.int16), Yd.cpu().view(torch.int16))
+                Y_o = oracle.forward(f64(l["X"][c]), oracle.bf16_round(l["P"]), f64(l["W"]))[0]
+                assert_y_close(l["Y"][c], Y_o)
+    finally:
+        for l in layers:
+            esp.espace_proj_destroy(l["p"])
+
+
 def test_linear_forward_full_rank_equals_dense_within_bf16(esp):
     """L = K: P P^T = I, so the projected layer reproduces the dense one (Sec. 2.2)."""
     N, K, M = 64, 256, 384
