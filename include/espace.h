@@ -318,8 +318,8 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
                                void* stream);
 
 /* Async. espace_linear_forward_host without the final wait: the copies and products are
- * queued as described there, the caller's stream is ordered after the last copy out, and the
- * call returns. X_host must not change, and Y_host is not filled, until the caller's stream
+ * queued as described there (in up to 8 chunks of at least 8192 tokens), the caller's stream
+ * is ordered after the last copy out, and the call returns. X_host must not change, and Y_host is not filled, until the caller's stream
  * reaches that point (synchronize it, or an event recorded on it after the call). Calls on
  * one handle must be ordered on one stream (they share the handle's staging); independent
  * layers on separate streams overlap one layer's copies with another's products. The first

@@ -259,7 +259,8 @@ def test_linear_forward_host_async_two_layers_on_two_streams(esp):
     its staging, so it must run after the first), nothing waited for until both streams are
     synchronized; every output equals the device-buffer forward bit for bit, and the oracle
     within the tolerances."""
-    shapes = [(1024, 1000, 512, 2304), (1536, 1000, 448, 1300)]   # K < 2 M: the fused kernel
+    # K < 2 M: the fused kernel; 16,500 tokens: two chunks (8448 + 8052), 1300: one
+    shapes = [(1024, 1000, 512, 16500), (1536, 1000, 448, 1300)]
     layers = []
     try:
         for i, (K, M, L, N) in enumerate(shapes):
