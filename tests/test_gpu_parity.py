@@ -978,6 +978,44 @@ def test_fused_forward_completes_while_other_work_holds_half_the_sms(esp):
         esp.espace_proj_destroy(p)
 
 
+@pytest.mark.parametrize("N", [64, 200])
+def test_few_token_forward_completes_while_other_work_holds_half_the_sms(esp, N):
+    """The few-token products are launches whose CTAs never wait for one another (each item's
+    tile, or split partial, is the CTA's own; the partials are added by the next launch). With
+    half of the SMs held by another stream's kernel (300 ms) they run on the other half
+    within a 50 ms wait limit and give the right result, for the projected layer and for the
+    dense one."""
+    K, M, L = 2048, 2048, 1024
+    p, Xd, Y_o = _layer_and_reference(esp, K, M, L, N, seed=81)
+    try:
+        Y = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_linear_forward(p, Xd, Y)            # workspace allocated here
+        W = dev(synth.weights(M, K, seed=81))
+        Yd = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+        esp.espace_dense_forward(Xd, W, Yd)
+        torch.cuda.synchronize()
+        esp.espace_check()
+        Y.fill_(float("nan"))
+        Yd.fill_(float("nan"))
+        sms = torch.cuda.get_device_properties(0).multi_processor_count
+        side = torch.cuda.Stream()
+        torch.cuda.synchronize()
+        esp.espace_set_wait_limit_ns(50_000_000)
+        try:
+            esp.espace_debug_occupy(sms // 2, 300_000_000, side)
+            time.sleep(0.02)                            # the holding CTAs are resident
+            esp.espace_linear_forward(p, Xd, Y)
+            esp.espace_dense_forward(Xd, W, Yd)
+            torch.cuda.synchronize()
+        finally:
+            esp.espace_set_wait_limit_ns(4_000_000_000)
+        esp.espace_check()                              # no wait gave up
+        assert_y_close(Y, Y_o)
+        assert_y_close(Yd, oracle.dense(f64(Xd.cpu()), f64(W.cpu())))
+    finally:
+        esp.espace_proj_destroy(p)
+
+
 @pytest.mark.parametrize("N", [1, 8, 24])
 def test_decode_forward_completes_while_other_work_holds_half_the_sms(esp, N):
     """The decode kernel's two products meet at a grid barrier, so it is a cooperative
@@ -1018,13 +1056,16 @@ def test_decode_forward_completes_while_other_work_holds_half_the_sms(esp, N):
         esp.espace_proj_destroy(p)
 
 
-@pytest.mark.parametrize("N,K,L", [(2048, 1024, 512), (4, 1024, 512), (4, 2048, 1536)])
+@pytest.mark.parametrize("N,K,L", [(2048, 1024, 512), (4, 1024, 512), (4, 2048, 1536), (64, 1024, 512),
+                                   (200, 2048, 1024)])
 def test_forward_after_a_launch_that_gave_up(esp, N, K, L):
     """A launch whose waits give up (a 2 us limit) leaves the handle's counters consistent:
     the fused kernel's last CTA zeroes its readiness counters, ticket and exit counter on
-    every exit path, and every CTA of the decode kernel arrives once at its grid barrier
-    (whose second phase runs over one k-block of Z at L = 512, two at L = 1536). The timeout
-    is reported, and the next forwards on the same handle are right."""
+    every exit path, every CTA of the decode kernel arrives once at its grid barrier (whose
+    second phase runs over one k-block of Z at L = 512, two at L = 1536), and the few-token
+    products (64 and 200 tokens: swapped launches with split reductions) keep no state
+    between launches. The timeout is reported, and the next forwards on the same handle are
+    right."""
     M = 2048
     p, Xd, Y_o = _layer_and_reference(esp, K, M, L, N, seed=78)
     try:
@@ -1039,14 +1080,14 @@ def test_forward_after_a_launch_that_gave_up(esp, N, K, L):
             torch.cuda.synchronize()
         finally:
             esp.espace_set_wait_limit_ns(4_000_000_000)
-        if N > 32:
+        if N > 256:
             with pytest.raises(esp.EspaceError) as e:
                 esp.espace_check()
             assert e.value.code == 5
         else:
             try:
                 esp.espace_check()
-            except esp.EspaceError as e:                # the short launch may finish in time
+            except esp.EspaceError as e:                # a short launch may finish in time
                 assert e.code == 5
         for _ in range(2):
             Y.fill_(float("nan"))
