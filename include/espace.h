@@ -329,6 +329,26 @@ int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, v
 int espace_linear_forward_host_async(espace_proj_t p, const void* X_host, int64_t N, void* Y_host,
                                      void* stream);
 
+/* Synchronous. The host-buffer forward of several independent layers in one pipeline:
+ * layer i (handle layers[i]) maps X_host[i] ([N[i]][K_i] bf16) to Y_host[i] ([N[i]][M_i]
+ * bf16) with the products of espace_linear_forward. The handles must be distinct and on
+ * one device. Every copy in runs on one copy stream and every product on the caller's
+ * stream, both in layer order, in token chunks of at least 8192. Every copy out runs on a
+ * second copy stream, so layer i + 1's tokens are copied in while layer i computes and layer
+ * i's outputs are copied out while layer i + 1 computes, with one product running at a
+ * time. Pinned host buffers let the copies overlap; pageable ones still give the right
+ * result. Work already on the caller's stream runs first; the call returns with every
+ * Y_host[i] filled. count <= ESPACE_HOST_MANY_MAX, and N[i] = 0 skips layer i. A handle's
+ * first call with a larger N than any before allocates its staging, as
+ * espace_linear_forward_host does. Errors (nothing is queued):
+ *   ESPACE_ERR_ARG for null arrays, handles or buffers, a repeated handle, or handles on
+ *     different devices;
+ *   ESPACE_ERR_STATE for a tensor-parallel handle;
+ *   ESPACE_ERR_SHAPE for a bad N[i]. */
+#define ESPACE_HOST_MANY_MAX 16
+int espace_linear_forward_host_many(int count, const espace_proj_t* layers, const void* const* X_host,
+                                    const int64_t* N, void* const* Y_host, void* stream);
+
 /* Capacity, in bf16 values, of the fixed scratch used by espace_linear_forward_noalloc:
  * 16 MiB, enough for N * Lp <= 8,388,608 (e.g. 4096 tokens at L = 2048). */
 #define ESPACE_NOALLOC_Z_ELEMS 8388608

@@ -36,6 +36,7 @@ __all__ = [
     "TP_COLUMN", "TP_ROW", "espace_proj_tp_from_host", "espace_build_projection_tp", "espace_proj_tp_info",
     "espace_calib_accumulate_nl", "espace_proj_refold", "espace_train_forward", "espace_train_backward",
     "espace_train_weight_grad", "espace_linear_forward_host", "espace_linear_forward_host_async",
+    "espace_linear_forward_host_many",
     "espace_dense_backward",
     "espace_linear_forward_launches",
 ]
@@ -101,6 +102,7 @@ _SIGNATURES = {
     "espace_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_linear_forward_host": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
     "espace_linear_forward_host_async": (ctypes.c_int, [_vp, _vp, _i64, _vp, _vp]),
+    "espace_linear_forward_host_many": (ctypes.c_int, [ctypes.c_int, _vp, _vp, _vp, _vp, _vp]),
     "espace_linear_forward_launches": (ctypes.c_int, [_vp, _i64, ctypes.c_int]),
     "espace_dense_forward": (ctypes.c_int, [_vp, _i64, _i64, _vp, _i64, _vp, _vp]),
     "espace_proj_refold": (ctypes.c_int, [_vp, _vp, _vp]),
@@ -401,6 +403,19 @@ def espace_linear_forward_host_async(p: int, X, Y, stream=None) -> None:
     only when the stream has passed this point."""
     _check(lib.espace_linear_forward_host_async(p, _host_ptr(X), int(X.shape[0]), _host_ptr(Y),
                                                 _stream(stream)))
+
+
+def espace_linear_forward_host_many(layers, Xs, Ys, stream=None) -> None:
+    """Several independent layers from host buffers in one pipeline: layers[i] maps the host
+    bf16 tensor Xs[i] [N_i][K_i] into Ys[i] [N_i][M_i] (pinned for overlapped copies)."""
+    n = len(layers)
+    if len(Xs) != n or len(Ys) != n:
+        raise ValueError("layers, Xs and Ys must have the same length")
+    hs = (ctypes.c_void_p * max(n, 1))(*[int(h) for h in layers])
+    xs = (ctypes.c_void_p * max(n, 1))(*[_host_ptr(x) for x in Xs])
+    ys = (ctypes.c_void_p * max(n, 1))(*[_host_ptr(y) for y in Ys])
+    ns = (ctypes.c_int64 * max(n, 1))(*[int(x.shape[0]) for x in Xs])
+    _check(lib.espace_linear_forward_host_many(n, hs, xs, ns, ys, _stream(stream)))
 
 
 def espace_linear_forward_noalloc(p: int, X, Y, N: int | None = None, stream=None) -> None:

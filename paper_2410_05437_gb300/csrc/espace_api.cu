@@ -1167,6 +1167,43 @@ static int host_chunks(int64_t N, int64_t min_chunk, int64_t* chunk)
 
 // The host-buffer forward; wait: return only once Y_host is filled (else the caller's stream
 // is ordered after the last copy out and the call returns once everything is queued).
+// The handle's copy streams, events and device staging for N tokens (created or grown on
+// first need; growth synchronizes the caller's stream).
+static int ensure_host_io(espace_proj_s* p, int64_t N, cudaStream_t st)
+{
+    std::lock_guard<std::mutex> lock(p->mu);
+    if (p->s_in == nullptr) {
+        cudaError_t e = cudaStreamCreateWithFlags(&p->s_in, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p->s_out, cudaStreamNonBlocking);
+        for (cudaEvent_t& ev : p->ev)
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) {
+            // release what was made, so that the next call starts over
+            for (cudaEvent_t& ev : p->ev)
+                if (ev) {
+                    cudaEventDestroy(ev);
+                    ev = nullptr;
+                }
+            if (p->s_out) cudaStreamDestroy(p->s_out);
+            if (p->s_in) cudaStreamDestroy(p->s_in);
+            p->s_in = p->s_out = nullptr;
+            return fail_cuda(e, "espace_linear_forward_host: streams");
+        }
+    }
+    if (p->h_cap < N) {
+        CUDA_TRY(cudaStreamSynchronize(st), "espace_linear_forward_host: sync before staging growth");
+        if (p->hx) cudaFree(p->hx);
+        if (p->hy) cudaFree(p->hy);
+        p->hx = p->hy = nullptr;
+        p->h_cap = 0;
+        cudaError_t e = cudaMalloc(&p->hx, sizeof(uint16_t) * N * p->K);
+        if (e == cudaSuccess) e = cudaMalloc(&p->hy, sizeof(uint16_t) * N * p->M);
+        if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_linear_forward_host: staging: %s", cudaGetErrorString(e));
+        p->h_cap = N;
+    }
+    return ESPACE_OK;
+}
+
 static int forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream, bool wait)
 {
     if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward_host: null handle");
@@ -1178,36 +1215,8 @@ static int forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int64_t K = p->K, M = p->M;
     {
-        std::lock_guard<std::mutex> lock(p->mu);
-        if (p->s_in == nullptr) {
-            cudaError_t e = cudaStreamCreateWithFlags(&p->s_in, cudaStreamNonBlocking);
-            if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p->s_out, cudaStreamNonBlocking);
-            for (cudaEvent_t& ev : p->ev)
-                if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
-            if (e != cudaSuccess) {
-                // release what was made, so that the next call starts over
-                for (cudaEvent_t& ev : p->ev)
-                    if (ev) {
-                        cudaEventDestroy(ev);
-                        ev = nullptr;
-                    }
-                if (p->s_out) cudaStreamDestroy(p->s_out);
-                if (p->s_in) cudaStreamDestroy(p->s_in);
-                p->s_in = p->s_out = nullptr;
-                return fail_cuda(e, "espace_linear_forward_host: streams");
-            }
-        }
-        if (p->h_cap < N) {
-            CUDA_TRY(cudaStreamSynchronize(st), "espace_linear_forward_host: sync before staging growth");
-            if (p->hx) cudaFree(p->hx);
-            if (p->hy) cudaFree(p->hy);
-            p->hx = p->hy = nullptr;
-            p->h_cap = 0;
-            cudaError_t e = cudaMalloc(&p->hx, sizeof(uint16_t) * N * K);
-            if (e == cudaSuccess) e = cudaMalloc(&p->hy, sizeof(uint16_t) * N * M);
-            if (e != cudaSuccess) return fail(ESPACE_ERR_NOMEM, "espace_linear_forward_host: staging: %s", cudaGetErrorString(e));
-            p->h_cap = N;
-        }
+        const int rc = ensure_host_io(p, N, st);
+        if (rc != ESPACE_OK) return rc;
     }
     // chunks of at least 512 tokens for the synchronous form (one layer in flight: the copies
     // overlap only its own chunks' products), of at least 8192 for the asynchronous one
@@ -1262,6 +1271,87 @@ static int forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_
     CUDA_TRY(cudaEventRecord(end, p->s_out), "espace_linear_forward_host: event");
     CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host: order");
     if (wait) CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host: wait");
+    drain.armed = false;
+    return ESPACE_OK;
+}
+
+int espace_linear_forward_host_many(int count, const espace_proj_t* layers, const void* const* X_host,
+                                    const int64_t* N, void* const* Y_host, void* stream)
+{
+    const char* what = "espace_linear_forward_host_many";
+    if (count < 0 || count > ESPACE_HOST_MANY_MAX) return fail(ESPACE_ERR_ARG, "%s: count=%d", what, count);
+    if (count == 0) return ESPACE_OK;
+    if (layers == nullptr || X_host == nullptr || N == nullptr || Y_host == nullptr)
+        return fail(ESPACE_ERR_ARG, "%s: null array", what);
+    for (int i = 0; i < count; ++i) {
+        espace_proj_s* p = layers[i];
+        if (p == nullptr) return fail(ESPACE_ERR_ARG, "%s: null handle %d", what, i);
+        if (p->tp_kind != 0) return fail(ESPACE_ERR_STATE, "%s: layer %d is a tensor-parallel handle", what, i);
+        if (p->device != layers[0]->device) return fail(ESPACE_ERR_ARG, "%s: layers on different devices", what);
+        if (N[i] < 0 || N[i] > (int64_t(1) << 31) - 256) return fail(ESPACE_ERR_SHAPE, "%s: N[%d]=%lld", what, i, (long long)N[i]);
+        if (N[i] > 0 && (X_host[i] == nullptr || Y_host[i] == nullptr)) return fail(ESPACE_ERR_ARG, "%s: null buffer %d", what, i);
+        for (int j = 0; j < i; ++j)
+            if (layers[j] == p) return fail(ESPACE_ERR_ARG, "%s: handle %d repeated", what, i);
+    }
+    espace_proj_s* h0 = layers[0];
+    DeviceGuard g(h0->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    for (int i = 0; i < count; ++i) {
+        const int rc = ensure_host_io(layers[i], std::max<int64_t>(N[i], 1), st);
+        if (rc != ESPACE_OK) return rc;
+    }
+    // one copy-in stream and one copy-out stream (the first handle's) for every layer, in
+    // order, and every product on the caller's stream: the next layer's tokens are copied in
+    // while this one computes, and only one product runs at a time
+    cudaStream_t s_in = h0->s_in, s_out = h0->s_out;
+    cudaEvent_t start = h0->ev[32], end = h0->ev[33];
+    CUDA_TRY(cudaEventRecord(start, st), "espace_linear_forward_host_many: order");
+    CUDA_TRY(cudaStreamWaitEvent(s_in, start, 0), "espace_linear_forward_host_many: order");
+    CUDA_TRY(cudaStreamWaitEvent(s_out, start, 0), "espace_linear_forward_host_many: order");
+    struct Drain {
+        cudaStream_t a, b, c;
+        bool armed = true;
+        ~Drain()
+        {
+            if (!armed) return;
+            cudaStreamSynchronize(a);
+            cudaStreamSynchronize(b);
+            cudaStreamSynchronize(c);
+        }
+    } drain{s_in, st, s_out};
+    int64_t chunk[ESPACE_HOST_MANY_MAX];
+    int nchunks[ESPACE_HOST_MANY_MAX];
+    for (int i = 0; i < count; ++i) {
+        // chunks of at least 8192 tokens: the other layers' copies fill the gaps
+        nchunks[i] = N[i] > 0 ? host_chunks(N[i], 8192, &chunk[i]) : 0;
+        espace_proj_s* p = layers[i];
+        const uint16_t* xh = static_cast<const uint16_t*>(X_host[i]);
+        for (int j = 0; j < nchunks[i]; ++j) {
+            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
+            CUDA_TRY(cudaMemcpyAsync(p->hx + t0 * p->K, xh + t0 * p->K, sizeof(uint16_t) * n * p->K,
+                                     cudaMemcpyHostToDevice, s_in),
+                     "espace_linear_forward_host_many: copy in");
+            CUDA_TRY(cudaEventRecord(p->ev[j], s_in), "espace_linear_forward_host_many: event");
+        }
+    }
+    for (int i = 0; i < count; ++i) {
+        espace_proj_s* p = layers[i];
+        uint16_t* yh = static_cast<uint16_t*>(Y_host[i]);
+        for (int j = 0; j < nchunks[i]; ++j) {
+            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
+            CUDA_TRY(cudaStreamWaitEvent(st, p->ev[j], 0), "espace_linear_forward_host_many: order");
+            int rc = espace_linear_forward_path(p, p->hx + t0 * p->K, n, p->hy + t0 * p->M, st, ESPACE_PATH_AUTO);
+            if (rc != ESPACE_OK) return rc;
+            CUDA_TRY(cudaEventRecord(p->ev[16 + j], st), "espace_linear_forward_host_many: event");
+            CUDA_TRY(cudaStreamWaitEvent(s_out, p->ev[16 + j], 0), "espace_linear_forward_host_many: order");
+            CUDA_TRY(cudaMemcpyAsync(yh + t0 * p->M, p->hy + t0 * p->M, sizeof(uint16_t) * n * p->M,
+                                     cudaMemcpyDeviceToHost, s_out),
+                     "espace_linear_forward_host_many: copy out");
+        }
+    }
+    CUDA_TRY(cudaEventRecord(end, s_out), "espace_linear_forward_host_many: event");
+    CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host_many: order");
+    CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host_many: wait");
     drain.armed = false;
     return ESPACE_OK;
 }

@@ -292,6 +292,55 @@ def test_linear_forward_host_async_two_layers_on_two_streams(esp):
             esp.espace_proj_destroy(l["p"])
 
 
+def test_linear_forward_host_many_layers_in_one_pipeline(esp):
+    """Several independent layers through one host-buffer pipeline: one copy-in stream, the
+    products in layer order on the caller's stream, one copy-out stream. Every output equals
+    the device-buffer forward bit for bit (chunks of at least 8192 tokens all run the fused
+    kernel, whose per-token sums do not depend on the batch) and the oracle within the
+    tolerances. A layer with N = 0 is skipped, an empty list is a no-op, and a repeated
+    handle or more than 16 layers is refused before anything is queued."""
+    # 16,500 tokens: two chunks; 300 and 1 token: one chunk (swapped products, decode kernel)
+    shapes = [(1024, 1000, 512, 16500), (1536, 776, 448, 300), (512, 520, 256, 0), (1040, 264, 100, 1)]
+    layers = []
+    try:
+        for i, (K, M, L, N) in enumerate(shapes):
+            model = synth.ActivationModel(K, seed=6200 + i)
+            W = synth.weights(M, K, seed=6200 + i)
+            P = synth.random_projection(K, L, seed=6200 + i)
+            p = esp.espace_proj_from_host(P, dev(W))
+            X = model.sample(N).contiguous().pin_memory() if N > 0 else torch.empty((0, K), dtype=torch.bfloat16)
+            Y = torch.full((max(N, 1), M), float("nan"), dtype=torch.bfloat16).pin_memory()[:N]
+            layers.append({"p": p, "P": P, "W": W, "X": X, "Y": Y})
+        for rep in range(2):   # the second call reuses every handle's staging
+            for l in layers:
+                l["Y"].fill_(float("nan"))
+            esp.espace_linear_forward_host_many([l["p"] for l in layers], [l["X"] for l in layers],
+                                                [l["Y"] for l in layers])
+            esp.espace_check()
+            for l in layers:
+                N, M = l["Y"].shape
+                if N == 0:
+                    continue
+                Yd = torch.empty((N, M), dtype=torch.bfloat16, device="cuda")
+                esp.espace_linear_forward(l["p"], dev(l["X"]), Yd)
+                torch.cuda.synchronize()
+                assert torch.equal(l["Y"].view(torch.int16), Yd.cpu().view(torch.int16))
+                if rep == 0:
+                    Y_o = oracle.forward(f64(l["X"]), oracle.bf16_round(l["P"]), f64(l["W"]))[0]
+                    assert_y_close(l["Y"], Y_o)
+        esp.espace_linear_forward_host_many([], [], [])
+        with pytest.raises(esp.EspaceError) as e:
+            esp.espace_linear_forward_host_many([layers[0]["p"], layers[0]["p"]], [layers[0]["X"]] * 2,
+                                                [layers[0]["Y"]] * 2)
+        assert e.value.code == 1                        # ESPACE_ERR_ARG
+        with pytest.raises(esp.EspaceError) as e:
+            esp.espace_linear_forward_host_many([layers[3]["p"]] * 17, [layers[3]["X"]] * 17, [layers[3]["Y"]] * 17)
+        assert e.value.code == 1                        # ESPACE_ERR_ARG
+    finally:
+        for l in layers:
+            esp.espace_proj_destroy(l["p"])
+
+
 def test_linear_forward_full_rank_equals_dense_within_bf16(esp):
     """L = K: P P^T = I, so the projected layer reproduces the dense one (Sec. 2.2)."""
     N, K, M = 64, 256, 384
