@@ -1165,8 +1165,6 @@ static int host_chunks(int64_t N, int64_t min_chunk, int64_t* chunk)
     return nc;
 }
 
-// The host-buffer forward; wait: return only once Y_host is filled (else the caller's stream
-// is ordered after the last copy out and the call returns once everything is queued).
 // The handle's copy streams, events and device staging for N tokens (created or grown on
 // first need; growth synchronizes the caller's stream).
 static int ensure_host_io(espace_proj_s* p, int64_t N, cudaStream_t st)
@@ -1204,6 +1202,83 @@ static int ensure_host_io(espace_proj_s* p, int64_t N, cudaStream_t st)
     return ESPACE_OK;
 }
 
+// The host-buffer pipeline over `count` independent layers (distinct handles, validated by
+// the caller): every copy in on the first handle's copy-in stream and every product on the
+// caller's stream, both in layer order, each copy out on the first handle's copy-out stream
+// once its chunk is computed. Layer i's tokens go in chunks of at least min_chunk (up to 8),
+// through layer i's staging and events. wait: return once every Y_host is filled; else the
+// caller's stream is ordered after the last copy out and the call returns once queued.
+static int host_pipeline(int count, espace_proj_s* const* layers, const void* const* X_host, const int64_t* N,
+                         void* const* Y_host, cudaStream_t st, int64_t min_chunk, bool wait)
+{
+    espace_proj_s* h0 = layers[0];
+    DeviceGuard g(h0->device);
+    for (int i = 0; i < count; ++i) {
+        const int rc = ensure_host_io(layers[i], std::max<int64_t>(N[i], 1), st);
+        if (rc != ESPACE_OK) return rc;
+    }
+    cudaStream_t s_in = h0->s_in, s_out = h0->s_out;
+    cudaEvent_t start = h0->ev[32], end = h0->ev[33];
+    // the copies start after the work already on the caller's stream
+    CUDA_TRY(cudaEventRecord(start, st), "espace_linear_forward_host: order");
+    CUDA_TRY(cudaStreamWaitEvent(s_in, start, 0), "espace_linear_forward_host: order");
+    CUDA_TRY(cudaStreamWaitEvent(s_out, start, 0), "espace_linear_forward_host: order");
+    // on an error after copies were queued, wait for them before returning, so that no copy
+    // touches the caller's host buffers after the call
+    struct Drain {
+        cudaStream_t a, b, c;
+        bool armed = true;
+        ~Drain()
+        {
+            if (!armed) return;
+            cudaStreamSynchronize(a);
+            cudaStreamSynchronize(b);
+            cudaStreamSynchronize(c);
+        }
+    } drain{s_in, st, s_out};
+    int64_t chunk[ESPACE_HOST_MANY_MAX];
+    int nchunks[ESPACE_HOST_MANY_MAX];
+    for (int i = 0; i < count; ++i) {
+        espace_proj_s* p = layers[i];
+        nchunks[i] = N[i] > 0 ? host_chunks(N[i], min_chunk, &chunk[i]) : 0;
+        const uint16_t* xh = static_cast<const uint16_t*>(X_host[i]);
+        for (int j = 0; j < nchunks[i]; ++j) {
+            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
+            CUDA_TRY(cudaMemcpyAsync(p->hx + t0 * p->K, xh + t0 * p->K, sizeof(uint16_t) * n * p->K,
+                                     cudaMemcpyHostToDevice, s_in),
+                     "espace_linear_forward_host: copy in");
+            CUDA_TRY(cudaEventRecord(p->ev[j], s_in), "espace_linear_forward_host: event");   // chunk j in
+        }
+    }
+    for (int i = 0; i < count; ++i) {
+        espace_proj_s* p = layers[i];
+        uint16_t* yh = static_cast<uint16_t*>(Y_host[i]);
+        for (int j = 0; j < nchunks[i]; ++j) {
+            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
+            // chunk j's product runs once its tokens are on the device, while other chunks'
+            // tokens and outputs are copied
+            CUDA_TRY(cudaStreamWaitEvent(st, p->ev[j], 0), "espace_linear_forward_host: order");
+            int rc = espace_linear_forward_path(p, p->hx + t0 * p->K, n, p->hy + t0 * p->M, st, ESPACE_PATH_AUTO);
+            if (rc != ESPACE_OK) return rc;
+            CUDA_TRY(cudaEventRecord(p->ev[16 + j], st), "espace_linear_forward_host: event");   // chunk j done
+            CUDA_TRY(cudaStreamWaitEvent(s_out, p->ev[16 + j], 0), "espace_linear_forward_host: order");
+            CUDA_TRY(cudaMemcpyAsync(yh + t0 * p->M, p->hy + t0 * p->M, sizeof(uint16_t) * n * p->M,
+                                     cudaMemcpyDeviceToHost, s_out),
+                     "espace_linear_forward_host: copy out");
+        }
+    }
+    CUDA_TRY(cudaEventRecord(end, s_out), "espace_linear_forward_host: event");
+    CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host: order");
+    if (wait) CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host: wait");
+    drain.armed = false;
+    return ESPACE_OK;
+}
+
+// One layer through the pipeline. Chunks of at least 512 tokens for the synchronous form
+// (one layer in flight: the copies overlap only its own chunks' products), of at least 8192
+// for the asynchronous one (other layers in flight fill the gaps, and long chunks keep each
+// product efficient: three 16,384-token layers on three streams took 10.3-10.6 ms per step
+// in 2 chunks, 11.0-11.6 ms in 8).
 static int forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream, bool wait)
 {
     if (p == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward_host: null handle");
@@ -1211,68 +1286,8 @@ static int forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_
     if (N < 0 || N > (int64_t(1) << 31) - 256) return fail(ESPACE_ERR_SHAPE, "espace_linear_forward_host: N=%lld", (long long)N);
     if (N == 0) return ESPACE_OK;
     if (X_host == nullptr || Y_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward_host: null pointer");
-    DeviceGuard g(p->device);
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const int64_t K = p->K, M = p->M;
-    {
-        const int rc = ensure_host_io(p, N, st);
-        if (rc != ESPACE_OK) return rc;
-    }
-    // chunks of at least 512 tokens for the synchronous form (one layer in flight: the copies
-    // overlap only its own chunks' products), of at least 8192 for the asynchronous one
-    // (other layers in flight fill the gaps, and long chunks keep each product efficient:
-    // three 16,384-token layers on three streams took 10.3-10.6 ms per step in 2 chunks,
-    // 11.0-11.6 ms in 8, with some steps 2.5 times slower)
-    int64_t C = 0;
-    const int nc = host_chunks(N, wait ? 512 : 8192, &C);
-    cudaEvent_t* ev_in = p->ev;           // chunk j copied in
-    cudaEvent_t* ev_done = p->ev + 16;    // chunk j computed
-    cudaEvent_t start = p->ev[32], end = p->ev[33];
-    // the copies start after the work already on the caller's stream
-    CUDA_TRY(cudaEventRecord(start, st), "espace_linear_forward_host: order");
-    CUDA_TRY(cudaStreamWaitEvent(p->s_in, start, 0), "espace_linear_forward_host: order");
-    CUDA_TRY(cudaStreamWaitEvent(p->s_out, start, 0), "espace_linear_forward_host: order");
-    const uint16_t* xh = static_cast<const uint16_t*>(X_host);
-    uint16_t* yh = static_cast<uint16_t*>(Y_host);
-    // on an error after copies were queued, wait for them before returning, so that no copy
-    // touches the caller's host buffers after the call
-    struct Drain {
-        espace_proj_s* p;
-        cudaStream_t st;
-        bool armed = true;
-        ~Drain()
-        {
-            if (!armed) return;
-            cudaStreamSynchronize(p->s_in);
-            cudaStreamSynchronize(st);
-            cudaStreamSynchronize(p->s_out);
-        }
-    } drain{p, st};
-    for (int j = 0; j < nc; ++j) {
-        const int64_t t0 = j * C, n = std::min(C, N - t0);
-        CUDA_TRY(cudaMemcpyAsync(p->hx + t0 * K, xh + t0 * K, sizeof(uint16_t) * n * K, cudaMemcpyHostToDevice, p->s_in),
-                 "espace_linear_forward_host: copy in");
-        CUDA_TRY(cudaEventRecord(ev_in[j], p->s_in), "espace_linear_forward_host: event");
-    }
-    for (int j = 0; j < nc; ++j) {
-        const int64_t t0 = j * C, n = std::min(C, N - t0);
-        // chunk j's product runs on the caller's stream once its tokens are on the device,
-        // while the next chunk's tokens and the previous chunk's outputs are copied
-        CUDA_TRY(cudaStreamWaitEvent(st, ev_in[j], 0), "espace_linear_forward_host: order");
-        int rc = espace_linear_forward_path(p, p->hx + t0 * K, n, p->hy + t0 * M, st, ESPACE_PATH_AUTO);
-        if (rc != ESPACE_OK) return rc;
-        CUDA_TRY(cudaEventRecord(ev_done[j], st), "espace_linear_forward_host: event");
-        CUDA_TRY(cudaStreamWaitEvent(p->s_out, ev_done[j], 0), "espace_linear_forward_host: order");
-        CUDA_TRY(cudaMemcpyAsync(yh + t0 * M, p->hy + t0 * M, sizeof(uint16_t) * n * M, cudaMemcpyDeviceToHost, p->s_out),
-                 "espace_linear_forward_host: copy out");
-    }
-    // the caller's stream continues after the last copy; the synchronous form returns with
-    // Y_host filled
-    CUDA_TRY(cudaEventRecord(end, p->s_out), "espace_linear_forward_host: event");
-    CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host: order");
-    if (wait) CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host: wait");
-    drain.armed = false;
-    return ESPACE_OK;
+    void* y = Y_host;
+    return host_pipeline(1, &p, &X_host, &N, &y, static_cast<cudaStream_t>(stream), wait ? 512 : 8192, wait);
 }
 
 int espace_linear_forward_host_many(int count, const espace_proj_t* layers, const void* const* X_host,
@@ -1293,67 +1308,8 @@ int espace_linear_forward_host_many(int count, const espace_proj_t* layers, cons
         for (int j = 0; j < i; ++j)
             if (layers[j] == p) return fail(ESPACE_ERR_ARG, "%s: handle %d repeated", what, i);
     }
-    espace_proj_s* h0 = layers[0];
-    DeviceGuard g(h0->device);
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    for (int i = 0; i < count; ++i) {
-        const int rc = ensure_host_io(layers[i], std::max<int64_t>(N[i], 1), st);
-        if (rc != ESPACE_OK) return rc;
-    }
-    // one copy-in stream and one copy-out stream (the first handle's) for every layer, in
-    // order, and every product on the caller's stream: the next layer's tokens are copied in
-    // while this one computes, and only one product runs at a time
-    cudaStream_t s_in = h0->s_in, s_out = h0->s_out;
-    cudaEvent_t start = h0->ev[32], end = h0->ev[33];
-    CUDA_TRY(cudaEventRecord(start, st), "espace_linear_forward_host_many: order");
-    CUDA_TRY(cudaStreamWaitEvent(s_in, start, 0), "espace_linear_forward_host_many: order");
-    CUDA_TRY(cudaStreamWaitEvent(s_out, start, 0), "espace_linear_forward_host_many: order");
-    struct Drain {
-        cudaStream_t a, b, c;
-        bool armed = true;
-        ~Drain()
-        {
-            if (!armed) return;
-            cudaStreamSynchronize(a);
-            cudaStreamSynchronize(b);
-            cudaStreamSynchronize(c);
-        }
-    } drain{s_in, st, s_out};
-    int64_t chunk[ESPACE_HOST_MANY_MAX];
-    int nchunks[ESPACE_HOST_MANY_MAX];
-    for (int i = 0; i < count; ++i) {
-        // chunks of at least 8192 tokens: the other layers' copies fill the gaps
-        nchunks[i] = N[i] > 0 ? host_chunks(N[i], 8192, &chunk[i]) : 0;
-        espace_proj_s* p = layers[i];
-        const uint16_t* xh = static_cast<const uint16_t*>(X_host[i]);
-        for (int j = 0; j < nchunks[i]; ++j) {
-            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
-            CUDA_TRY(cudaMemcpyAsync(p->hx + t0 * p->K, xh + t0 * p->K, sizeof(uint16_t) * n * p->K,
-                                     cudaMemcpyHostToDevice, s_in),
-                     "espace_linear_forward_host_many: copy in");
-            CUDA_TRY(cudaEventRecord(p->ev[j], s_in), "espace_linear_forward_host_many: event");
-        }
-    }
-    for (int i = 0; i < count; ++i) {
-        espace_proj_s* p = layers[i];
-        uint16_t* yh = static_cast<uint16_t*>(Y_host[i]);
-        for (int j = 0; j < nchunks[i]; ++j) {
-            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
-            CUDA_TRY(cudaStreamWaitEvent(st, p->ev[j], 0), "espace_linear_forward_host_many: order");
-            int rc = espace_linear_forward_path(p, p->hx + t0 * p->K, n, p->hy + t0 * p->M, st, ESPACE_PATH_AUTO);
-            if (rc != ESPACE_OK) return rc;
-            CUDA_TRY(cudaEventRecord(p->ev[16 + j], st), "espace_linear_forward_host_many: event");
-            CUDA_TRY(cudaStreamWaitEvent(s_out, p->ev[16 + j], 0), "espace_linear_forward_host_many: order");
-            CUDA_TRY(cudaMemcpyAsync(yh + t0 * p->M, p->hy + t0 * p->M, sizeof(uint16_t) * n * p->M,
-                                     cudaMemcpyDeviceToHost, s_out),
-                     "espace_linear_forward_host_many: copy out");
-        }
-    }
-    CUDA_TRY(cudaEventRecord(end, s_out), "espace_linear_forward_host_many: event");
-    CUDA_TRY(cudaStreamWaitEvent(st, end, 0), "espace_linear_forward_host_many: order");
-    CUDA_TRY(cudaEventSynchronize(end), "espace_linear_forward_host_many: wait");
-    drain.armed = false;
-    return ESPACE_OK;
+    // chunks of at least 8192 tokens: the other layers' copies fill the gaps
+    return host_pipeline(count, layers, X_host, N, Y_host, static_cast<cudaStream_t>(stream), 8192, true);
 }
 
 int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream)
