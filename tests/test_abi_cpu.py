@@ -85,6 +85,10 @@ def test_null_handles_and_pointers_are_refused_without_gpu():
         "espace_linear_forward_path": lambda: L.espace_linear_forward_path(None, x, 8, x, None, 0),
         "espace_linear_forward_noalloc": lambda: L.espace_linear_forward_noalloc(None, x, 8, x, None),
         "espace_linear_forward_host": lambda: L.espace_linear_forward_host(None, x, 8, x, None),
+        "espace_linear_forward_host_async": lambda: L.espace_linear_forward_host_async(None, x, 8, x, None),
+        "espace_linear_forward_host_many": lambda: L.espace_linear_forward_host_many(
+            1, (ctypes.c_void_p * 1)(None), (ctypes.c_void_p * 1)(x), (ctypes.c_int64 * 1)(8),
+            (ctypes.c_void_p * 1)(x), None),
         "espace_proj_refold": lambda: L.espace_proj_refold(None, x, None),
         "espace_train_forward": lambda: L.espace_train_forward(None, x, 8, x, x, None),
         "espace_train_backward": lambda: L.espace_train_backward(None, x, x, 8, x, None),
@@ -100,6 +104,12 @@ def test_null_handles_and_pointers_are_refused_without_gpu():
     assert L.espace_dense_forward(x, 8, 12, x, 64, x, None) == 2           # K not a multiple of 8
     odd = ctypes.c_void_p(264)                                              # 8-byte aligned only
     assert L.espace_dense_forward(odd, 8, 64, x, 64, x, None) == 3          # ESPACE_ERR_ALIGN
+    # several layers through one pipeline: the count and the arrays are checked first
+    arr = (ctypes.c_void_p * 1)(x)
+    assert L.espace_linear_forward_host_many(0, None, None, None, None, None) == 0   # nothing to do
+    assert L.espace_linear_forward_host_many(-1, arr, arr, (ctypes.c_int64 * 1)(8), arr, None) == 1
+    assert L.espace_linear_forward_host_many(17, arr, arr, (ctypes.c_int64 * 1)(8), arr, None) == 1
+    assert L.espace_linear_forward_host_many(1, None, arr, (ctypes.c_int64 * 1)(8), arr, None) == 1
 
 
 @pytest.mark.parametrize("K", [1, 2, 9, 64, 200])
