@@ -333,10 +333,11 @@ int espace_linear_forward_host_async(espace_proj_t p, const void* X_host, int64_
  * layer i (handle layers[i]) maps X_host[i] ([N[i]][K_i] bf16) to Y_host[i] ([N[i]][M_i]
  * bf16) with the products of espace_linear_forward. The handles must be distinct and on
  * one device. Every copy in runs on one copy stream and every product on the caller's
- * stream, both in layer order, in token chunks of at least 8192. Every copy out runs on a
- * second copy stream, so layer i + 1's tokens are copied in while layer i computes and layer
- * i's outputs are copied out while layer i + 1 computes, with one product running at a
- * time. Pinned host buffers let the copies overlap; pageable ones still give the right
+ * stream, both in layer order, in token chunks of about 8192 (up to 8 per layer). The first
+ * layer leads with chunks of 2048 and 4096 tokens, and the last layer ends with one of 2048,
+ * where N leaves room. Every copy out runs on a second copy stream, so layer i + 1's tokens
+ * are copied in while layer i computes and layer i's outputs are copied out while layer
+ * i + 1 computes, with one product running at a time. Pinned host buffers let the copies overlap; pageable ones still give the right
  * result. Work already on the caller's stream runs first; the call returns with every
  * Y_host[i] filled. count <= ESPACE_HOST_MANY_MAX, and N[i] = 0 skips layer i. A handle's
  * first call with a larger N than any before allocates its staging, as

@@ -1202,12 +1202,43 @@ static int ensure_host_io(espace_proj_s* p, int64_t N, cudaStream_t st)
     return ESPACE_OK;
 }
 
+// Chunk boundaries (b[0] = 0 < ... < b[n] = N, n <= 11) of one layer's N tokens in the
+// pipeline of several layers: up to 8 chunks of about 8192 tokens (at most, below 64K
+// tokens); the pipeline's first layer leads with chunks of 2048 and 4096 tokens (its first
+// product starts once 2048 tokens are in, and each next chunk is copied in while the one
+// before computes), and its last layer ends with a 2048-token chunk (the last copy out is
+// short), where N leaves room for them.
+static int many_bounds(int64_t N, bool first, bool last, int64_t* b)
+{
+    if (N <= 0) return 0;
+    int n = 0;
+    b[0] = 0;
+    int64_t lo = 0;
+    const int64_t keep = 8192 + (last ? 2048 : 0);
+    if (first)
+        for (int64_t h : {int64_t(2048), int64_t(4096)})
+            if (N - lo >= h + keep) {
+                lo += h;
+                b[++n] = lo;
+            }
+    const int64_t tail = (last && N - lo >= 2048 + 8192) ? 2048 : 0;
+    const int64_t hi = N - tail;
+    const int64_t k = std::min<int64_t>(8, (hi - lo + 8191) / 8192);
+    int64_t c = (hi - lo + k - 1) / k;
+    c = (c + 255) / 256 * 256;
+    for (int64_t t = lo + c; t < hi; t += c) b[++n] = t;
+    b[++n] = hi;
+    if (tail > 0) b[++n] = N;
+    return n;
+}
+
 // The host-buffer pipeline over `count` independent layers (distinct handles, validated by
 // the caller): every copy in on the first handle's copy-in stream and every product on the
 // caller's stream, both in layer order, each copy out on the first handle's copy-out stream
-// once its chunk is computed. Layer i's tokens go in chunks of at least min_chunk (up to 8),
-// through layer i's staging and events. wait: return once every Y_host is filled; else the
-// caller's stream is ordered after the last copy out and the call returns once queued.
+// once its chunk is computed, through layer i's staging and events. One layer alone goes in
+// chunks of at least min_chunk (up to 8); several go in the chunks of many_bounds. wait:
+// return once every Y_host is filled; else the caller's stream is ordered after the last
+// copy out and the call returns once queued.
 static int host_pipeline(int count, espace_proj_s* const* layers, const void* const* X_host, const int64_t* N,
                          void* const* Y_host, cudaStream_t st, int64_t min_chunk, bool wait)
 {
@@ -1236,14 +1267,20 @@ static int host_pipeline(int count, espace_proj_s* const* layers, const void* co
             cudaStreamSynchronize(c);
         }
     } drain{s_in, st, s_out};
-    int64_t chunk[ESPACE_HOST_MANY_MAX];
+    int64_t bounds[ESPACE_HOST_MANY_MAX][12];
     int nchunks[ESPACE_HOST_MANY_MAX];
     for (int i = 0; i < count; ++i) {
         espace_proj_s* p = layers[i];
-        nchunks[i] = N[i] > 0 ? host_chunks(N[i], min_chunk, &chunk[i]) : 0;
+        if (count == 1) {
+            int64_t c = 0;
+            nchunks[i] = N[i] > 0 ? host_chunks(N[i], min_chunk, &c) : 0;
+            for (int j = 0; j <= nchunks[i]; ++j) bounds[i][j] = std::min(j * c, N[i]);
+        } else {
+            nchunks[i] = many_bounds(N[i], i == 0, i == count - 1, bounds[i]);
+        }
         const uint16_t* xh = static_cast<const uint16_t*>(X_host[i]);
         for (int j = 0; j < nchunks[i]; ++j) {
-            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
+            const int64_t t0 = bounds[i][j], n = bounds[i][j + 1] - t0;
             CUDA_TRY(cudaMemcpyAsync(p->hx + t0 * p->K, xh + t0 * p->K, sizeof(uint16_t) * n * p->K,
                                      cudaMemcpyHostToDevice, s_in),
                      "espace_linear_forward_host: copy in");
@@ -1254,7 +1291,7 @@ static int host_pipeline(int count, espace_proj_s* const* layers, const void* co
         espace_proj_s* p = layers[i];
         uint16_t* yh = static_cast<uint16_t*>(Y_host[i]);
         for (int j = 0; j < nchunks[i]; ++j) {
-            const int64_t t0 = j * chunk[i], n = std::min(chunk[i], N[i] - t0);
+            const int64_t t0 = bounds[i][j], n = bounds[i][j + 1] - t0;
             // chunk j's product runs once its tokens are on the device, while other chunks'
             // tokens and outputs are copied
             CUDA_TRY(cudaStreamWaitEvent(st, p->ev[j], 0), "espace_linear_forward_host: order");
