@@ -1235,12 +1235,12 @@ static int many_bounds(int64_t N, bool first, bool last, int64_t* b)
 // The host-buffer pipeline over `count` independent layers (distinct handles, validated by
 // the caller): every copy in on the first handle's copy-in stream and every product on the
 // caller's stream, both in layer order, each copy out on the first handle's copy-out stream
-// once its chunk is computed, through layer i's staging and events. One layer alone goes in
-// chunks of at least min_chunk (up to 8); several go in the chunks of many_bounds. wait:
-// return once every Y_host is filled; else the caller's stream is ordered after the last
-// copy out and the call returns once queued.
+// once its chunk is computed, through layer i's staging and events. The layers' tokens go
+// in the chunks of many_bounds (several_layers), else in chunks of at least min_chunk (up
+// to 8). wait: return once every Y_host is filled; else the caller's stream is ordered after
+// the last copy out and the call returns once queued.
 static int host_pipeline(int count, espace_proj_s* const* layers, const void* const* X_host, const int64_t* N,
-                         void* const* Y_host, cudaStream_t st, int64_t min_chunk, bool wait)
+                         void* const* Y_host, cudaStream_t st, int64_t min_chunk, bool wait, bool several_layers)
 {
     espace_proj_s* h0 = layers[0];
     DeviceGuard g(h0->device);
@@ -1271,12 +1271,12 @@ static int host_pipeline(int count, espace_proj_s* const* layers, const void* co
     int nchunks[ESPACE_HOST_MANY_MAX];
     for (int i = 0; i < count; ++i) {
         espace_proj_s* p = layers[i];
-        if (count == 1) {
+        if (several_layers) {
+            nchunks[i] = many_bounds(N[i], i == 0, i == count - 1, bounds[i]);
+        } else {
             int64_t c = 0;
             nchunks[i] = N[i] > 0 ? host_chunks(N[i], min_chunk, &c) : 0;
             for (int j = 0; j <= nchunks[i]; ++j) bounds[i][j] = std::min(j * c, N[i]);
-        } else {
-            nchunks[i] = many_bounds(N[i], i == 0, i == count - 1, bounds[i]);
         }
         const uint16_t* xh = static_cast<const uint16_t*>(X_host[i]);
         for (int j = 0; j < nchunks[i]; ++j) {
@@ -1324,7 +1324,7 @@ static int forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_
     if (N == 0) return ESPACE_OK;
     if (X_host == nullptr || Y_host == nullptr) return fail(ESPACE_ERR_ARG, "espace_linear_forward_host: null pointer");
     void* y = Y_host;
-    return host_pipeline(1, &p, &X_host, &N, &y, static_cast<cudaStream_t>(stream), wait ? 512 : 8192, wait);
+    return host_pipeline(1, &p, &X_host, &N, &y, static_cast<cudaStream_t>(stream), wait ? 512 : 8192, wait, false);
 }
 
 int espace_linear_forward_host_many(int count, const espace_proj_t* layers, const void* const* X_host,
@@ -1345,8 +1345,8 @@ int espace_linear_forward_host_many(int count, const espace_proj_t* layers, cons
         for (int j = 0; j < i; ++j)
             if (layers[j] == p) return fail(ESPACE_ERR_ARG, "%s: handle %d repeated", what, i);
     }
-    // chunks of at least 8192 tokens: the other layers' copies fill the gaps
-    return host_pipeline(count, layers, X_host, N, Y_host, static_cast<cudaStream_t>(stream), 8192, true);
+    // the chunks of many_bounds: about 8192 tokens, shorter at the pipeline's two ends
+    return host_pipeline(count, layers, X_host, N, Y_host, static_cast<cudaStream_t>(stream), 8192, true, true);
 }
 
 int espace_linear_forward_host(espace_proj_t p, const void* X_host, int64_t N, void* Y_host, void* stream)
