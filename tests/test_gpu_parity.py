@@ -295,11 +295,12 @@ def test_linear_forward_host_async_two_layers_on_two_streams(esp):
 def test_linear_forward_host_many_layers_in_one_pipeline(esp):
     """Several independent layers through one host-buffer pipeline: one copy-in stream, the
     products in layer order on the caller's stream, one copy-out stream. Every output equals
-    the device-buffer forward bit for bit (chunks of at least 8192 tokens all run the fused
+    the device-buffer forward bit for bit (chunks of at least 2048 tokens all run the fused
     kernel, whose per-token sums do not depend on the batch) and the oracle within the
     tolerances. A layer with N = 0 is skipped, an empty list is a no-op, and a repeated
     handle or more than 16 layers is refused before anything is queued."""
-    # 16,500 tokens: two chunks; 300 and 1 token: one chunk (swapped products, decode kernel)
+    # 16,500 tokens, the first layer: chunks of 2048, 4096, 5376 and 4980 tokens; 300 and 1
+    # token: one chunk each (the fused launch, the decode kernel)
     shapes = [(1024, 1000, 512, 16500), (1536, 776, 448, 300), (512, 520, 256, 0), (1040, 264, 100, 1)]
     layers = []
     try:
